@@ -1,0 +1,25 @@
+import os
+import sys
+
+import pytest
+
+REPO = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if REPO not in sys.path:
+    sys.path.insert(0, REPO)
+
+
+def pytest_configure(config):
+    config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300, sm_103a)")
+    config.addinivalue_line("markers", "slow: long-running on CPU")
+
+
+@pytest.fixture(scope="session")
+def tiny_workload():
+    from synth.workloads import TINY
+    return TINY
+
+
+@pytest.fixture(scope="session")
+def tiny_oracle(tiny_workload):
+    import oracle
+    return oracle.Model(tiny_workload.shape)
