@@ -113,6 +113,9 @@ def lib():
             L.orc_sess_kv.restype = C.c_double
             L.orc_forward.argtypes = [p, p, i32, i32, i32, i32, p]
             L.orc_logits.argtypes = [p, p, p]
+            L.orc_matvec.argtypes = [p, i32, i32, p, p]
+            L.orc_matvec_synth.argtypes = [C.c_uint32, C.c_uint32, C.c_double, i32, C.c_int64,
+                                           C.c_int64, C.c_int64, p, p]
             L.orc_stats_from_logits.argtypes = [p, i32, i32, C.POINTER(Stats)]
             L.orc_stats_from_logits.restype = None
             L.orc_exit_head.argtypes = [p, p, p, i32, C.POINTER(Stats)]
@@ -219,6 +222,15 @@ class Model:
     def get(self, which: int, layer: int, idx: int) -> float:
         return lib().orc_model_get(self.h, which, layer, idx)
 
+    def matvec(self, which: int, layer: int, x) -> np.ndarray:
+        x = np.ascontiguousarray(x, dtype=np.float64)
+        rows = {T_EMBED: self.shape.vocab, T_LMHEAD: self.shape.vocab, T_WQKV: self.shape.qkv_rows,
+                T_WO: self.shape.d_model, T_WGU: 2 * self.shape.ffn_dim,
+                T_WDOWN: self.shape.d_model}[which]
+        y = np.zeros(rows, dtype=np.float64)
+        _check(lib().orc_matvec(self.h, which, layer, _ptr(x), _ptr(y)), "orc_matvec")
+        return y
+
     def logits(self, h) -> np.ndarray:
         h = np.ascontiguousarray(h, dtype=np.float64)
         z = np.zeros(self.shape.vocab, dtype=np.float64)
@@ -302,6 +314,14 @@ class Session:
         _check(lib().orc_generate(self.h, C.byref(policy), n_new, _ptr(out), logs, logs_cap,
                                   _ptr(nr)), "orc_generate")
         return out, [logs[i].as_dict() for i in range(min(int(nr[0]), logs_cap))]
+
+
+def matvec_synth(seed: int, tid: int, sigma: float, bf16: bool, row0: int, nrows: int, x) -> np.ndarray:
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    y = np.zeros(nrows, dtype=np.float64)
+    _check(lib().orc_matvec_synth(seed, tid, sigma, 1 if bf16 else 0, row0, nrows, x.size, _ptr(x),
+                                  _ptr(y)), "orc_matvec_synth")
+    return y
 
 
 def num_threads() -> int:

@@ -274,6 +274,45 @@ static void matvec(const tensor* W, int64_t row0, int64_t nrows, int64_t K, cons
   }
 }
 
+/* y = W x for one of the model's matrices (which = ORC_T_*, layer for the
+ * per-layer ones); x has the matrix's column count. */
+int orc_matvec(const orc_model* m, int which, int layer, const double* x, double* y) {
+  const orc_cfg* c = &m->c;
+  tensor* t = pick(m, which, layer);
+  if (!t) return ORC_ERR_ARG;
+  int64_t qd = (int64_t)c->n_heads * c->head_dim;
+  int64_t rows, cols;
+  switch (which) {
+    case ORC_T_EMBED:
+    case ORC_T_LMHEAD: rows = c->vocab; cols = c->d_model; break;
+    case ORC_T_WQKV: rows = qkv_rows(c); cols = c->d_model; break;
+    case ORC_T_WO: rows = c->d_model; cols = qd; break;
+    case ORC_T_WGU: rows = 2 * (int64_t)c->ffn_dim; cols = c->d_model; break;
+    default: rows = c->d_model; cols = c->ffn_dim; break;
+  }
+  matvec(t, 0, rows, cols, x, y);
+  return ORC_OK;
+}
+
+/* y[r] = sum_k W[row0 + r][k] x[k] for rows of a synthetic matrix whose
+ * element (i, k) is the generator's value for flat index i*K + k (bf16-rounded
+ * when bf16); lets full-size matrices be checked on sampled rows without
+ * materialising them. */
+int orc_matvec_synth(uint32_t seed, uint32_t tid, double sigma, int bf16, int64_t row0,
+                     int64_t nrows, int64_t K, const double* x, double* y) {
+#pragma omp parallel for schedule(static)
+  for (int64_t r = 0; r < nrows; ++r) {
+    double acc = 0.0;
+    for (int64_t k = 0; k < K; ++k) {
+      float w = synth_weight_f32(seed, tid, (uint64_t)((row0 + r) * K + k), sigma);
+      if (bf16) w = synth_bf16_to_f32(synth_f32_to_bf16(w));
+      acc += (double)w * x[k];
+    }
+    y[r] = acc;
+  }
+  return ORC_OK;
+}
+
 /* RMSNorm: out = x / sqrt(mean(x^2) + eps) * g. */
 static void rmsnorm(const double* x, const double* g, int d, double eps, double* out) {
   double ss = 0.0;

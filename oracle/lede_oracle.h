@@ -91,6 +91,9 @@ double orc_sess_kv(const orc_sess* s, int layer, int kv, int head, int pos, int 
 
 int orc_forward(orc_sess* s, const int32_t* tok, int M, int pos0, int l_from, int l_to, double* h);
 int orc_logits(const orc_model* m, const double* h, double* z);
+int orc_matvec(const orc_model* m, int which, int layer, const double* x, double* y);
+int orc_matvec_synth(uint32_t seed, uint32_t tid, double sigma, int bf16, int64_t row0,
+                     int64_t nrows, int64_t K, const double* x, double* y);
 void orc_stats_from_logits(const double* z, int V, int topk, orc_stats* st);
 int orc_exit_head(const orc_model* m, const double* h, double* z_opt, int topk, orc_stats* st);
 void orc_qnet(const float* params, int in, int hidden, const double* s, double q[2]);

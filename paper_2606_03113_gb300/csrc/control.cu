@@ -1,0 +1,410 @@
+// control.cu -- the device-side control flow of a speculation round: token
+// embedding, round set-up, the Q-network decision at a candidate exit layer or
+// after a draft, greedy acceptance with KV rollback and the C_trace window.
+// Decisions set CUDA-graph conditional handles, so the walk, the drafting loop
+// and the generation loop run without returning to the host.
+#include <math.h>
+
+#include "../../synth/synth.h"
+#include "kernels.h"
+
+namespace ssd {
+
+__device__ __forceinline__ void set_cond(cudaGraphConditionalHandle h, unsigned v) {
+  if (h) cudaGraphSetConditional(h, v);
+}
+
+__device__ __forceinline__ void trace_push(Ctl* c, float p) {
+  c->trace[c->trace_head] = p;
+  c->trace_head = (c->trace_head + 1) % kTraceCap;
+  if (c->trace_n < kTraceCap) ++c->trace_n;
+}
+
+// C_trace = -(1/n) sum log pmax over the n = min(T, count) most recent entries
+// (§3.1.1, average trace of token confidence).
+__device__ float trace_conf(const Ctl* c, int T) {
+  const int n = min(T, c->trace_n);
+  if (n <= 0) return 0.f;
+  float acc = 0.f;
+  for (int i = n; i >= 1; --i) acc += logf(c->trace[(c->trace_head - i + kTraceCap) % kTraceCap]);
+  return -acc / (float)n;
+}
+
+// h[m] = embed[token_m] (fp32) and the row's sum of squares for the first
+// RMSNorm.  One block per row.  Optionally sets the drafting switch handle to
+// the chosen exit-layer index.
+template <typename T>
+__global__ void k_embed(Dims D, Bufs B, const T* __restrict__ emb, RowSel sel,
+                        cudaGraphConditionalHandle sw) {
+  __shared__ float red[32];
+  Ctl* c = B.ctl;
+  int pos0, M;
+  resolve_rows(c, sel, pos0, M);
+  const int m = blockIdx.x;
+  if (blockIdx.x == 0 && threadIdx.x == 0) set_cond(sw, (unsigned)c->lstar_idx);
+  if (m >= M) return;
+  int tok;
+  switch (sel.mode) {
+    case kRowsWalk: tok = c->tok[0]; break;
+    case kRowsDraft: tok = c->tok[c->k]; break;
+    case kRowsVerify: tok = c->tok[m]; break;
+    default: tok = sel.tok[m]; break;
+  }
+  if (tok < 0 || tok >= D.V) {
+    if (threadIdx.x == 0) atomicOr(&c->err, (int)kErrToken);
+    tok = 0;
+  }
+  const T* row = emb + (size_t)tok * D.d;
+  float* hr = B.h + (size_t)m * D.d;
+  float ss = 0.f;
+  for (int i = threadIdx.x; i < D.d; i += blockDim.x) {
+    const float v = Elem<T>::to_f(row[i]);
+    hr[i] = v;
+    ss = fmaf(v, v, ss);
+  }
+  ss = warp_sum(ss);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float s = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s += red[w];
+    B.ss[m] = s;
+  }
+}
+
+// Draft cap of the round: min(kmax, tokens still to emit - 1), the static
+// length for a static policy, and the KV capacity.
+__global__ void k_round_begin(Dims D, Bufs B, cudaGraphConditionalHandle draft_if) {
+  Ctl* c = B.ctl;
+  const DevPolicy& P = c->pol;
+  const int remaining = c->max_new - c->n_out;
+  int kcap = 0;
+  if (P.kind != SSD_POLICY_AR) {
+    kcap = min(P.kmax, remaining - 1);
+    if (P.kind == SSD_POLICY_STATIC) kcap = min(kcap, P.static_k);
+  }
+  if (c->pos + kcap + 1 > D.max_seq) {
+    atomicOr(&c->err, (int)kErrCapacity);
+    kcap = max(0, D.max_seq - c->pos - 1);
+  }
+  kcap = max(kcap, 0);
+  c->kcap = kcap;
+  c->k = 0;
+  c->lstar = 0;
+  c->lstar_idx = 0;
+  c->keep = 0;
+  c->tok[0] = c->x;
+  ssd_round_trace& r = c->cur;
+  r.pos = c->pos;
+  r.x = c->x;
+  r.kcap = kcap;
+  r.n_visited = 0;
+  r.lstar = 0;
+  r.k = 0;
+  r.a = 0;
+  r.n_emit = 0;
+  r.n_q = 0;
+  set_cond(draft_if, kcap > 0 ? 1u : 0u);
+}
+
+// Decision at a candidate exit layer (walk) or after a draft (§3.1.2, §3.3).
+// LEDE: Q = W2 relu(W1 s + b1) + b2 on s = (C_k, H, C_trace) of the exit
+// distribution in stats[0]; greedy action, ties -> continue (0).
+//  walk:  exit (or the last candidate, forced) fixes l* and d_1 = argmax; the
+//         action itself says whether to keep drafting; continue opens the
+//         next walk segment (next_if).
+//  draft: record d_{k+1}; keep drafting while the action is exit and k < kcap.
+// Static policies exit at their only candidate and draft to their length.
+__global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, int layer,
+                         cudaGraphConditionalHandle next_if,
+                         cudaGraphConditionalHandle draft_while) {
+  __shared__ float s_state[3];
+  __shared__ float red0[32], red1[32];
+  Ctl* c = B.ctl;
+  const DevPolicy& P = c->pol;
+  const RowStats& st = B.stats[0];
+  const bool lede = P.kind == SSD_POLICY_LEDE;
+  const int tid = threadIdx.x;
+  float q0 = 0.f, q1 = 0.f;
+  if (lede) {
+    if (tid == 0) {
+      s_state[0] = st.conf_k;
+      s_state[1] = st.entropy;
+      s_state[2] = trace_conf(c, P.trace_T);
+    }
+    __syncthreads();
+    const int H = P.q_hidden;
+    const float* W1 = B.qparams;
+    const float* b1 = W1 + 3 * H;
+    const float* W2 = b1 + H;
+    const float* b2 = W2 + 2 * H;
+    float a0 = 0.f, a1 = 0.f;
+    for (int j = tid; j < H; j += blockDim.x) {
+      float z = b1[j];
+      z = fmaf(W1[3 * j], s_state[0], z);
+      z = fmaf(W1[3 * j + 1], s_state[1], z);
+      z = fmaf(W1[3 * j + 2], s_state[2], z);
+      const float r = fmaxf(z, 0.f);
+      a0 = fmaf(W2[j], r, a0);
+      a1 = fmaf(W2[H + j], r, a1);
+    }
+    a0 = warp_sum(a0);
+    a1 = warp_sum(a1);
+    if ((tid & 31) == 0) {
+      red0[tid >> 5] = a0;
+      red1[tid >> 5] = a1;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+        q0 += red0[w];
+        q1 += red1[w];
+      }
+      q0 += b2[0];
+      q1 += b2[1];
+    }
+  }
+  if (tid != 0) return;
+  ssd_round_trace& r = c->cur;
+  const int aq = lede ? (q1 > q0 ? 1 : 0) : 1;
+  if (lede && r.n_q < SSD_TRACE_MAXQ) {
+    const int i = r.n_q++;
+    r.q_action[i] = aq;
+    r.q_val[i][0] = q0;
+    r.q_val[i][1] = q1;
+    r.q_state[i][0] = s_state[0];
+    r.q_state[i][1] = s_state[1];
+    r.q_state[i][2] = s_state[2];
+  }
+  if (st.argmax < 0 || st.argmax >= D.V) atomicOr(&c->err, (int)kErrToken);
+  if (mode == kDecideWalk) {
+    if (r.n_visited < SSD_TRACE_MAXC) r.visited[r.n_visited++] = layer;
+    const int act = is_last ? 1 : aq;
+    if (act) {
+      c->lstar = layer;
+      c->lstar_idx = cand_idx;
+      c->k = 1;
+      c->tok[1] = st.argmax;
+      r.drafts[0] = st.argmax;
+      r.draft_margin[0] = st.margin;
+      c->keep = (aq && 1 < c->kcap) ? 1 : 0;
+      set_cond(next_if, 0u);
+    } else {
+      set_cond(next_if, 1u);
+    }
+  } else {
+    const int k = c->k;
+    if (k < 1 || k >= c->kcap || k >= kMaxDraft) {
+      atomicOr(&c->err, (int)kErrControl);
+      c->keep = 0;
+      set_cond(draft_while, 0u);
+      return;
+    }
+    c->tok[k + 1] = st.argmax;
+    r.drafts[k] = st.argmax;
+    r.draft_margin[k] = st.margin;
+    c->k = k + 1;
+    c->keep = (aq && k + 1 < c->kcap) ? 1 : 0;
+    set_cond(draft_while, (unsigned)c->keep);
+  }
+}
+
+__global__ void k_draft_begin(Bufs B, cudaGraphConditionalHandle draft_while) {
+  set_cond(draft_while, (unsigned)B.ctl->keep);
+}
+
+// Greedy verification (§4.1: greedy decoding, speculative acceptance):
+// g_i = argmax of verify row i; a = longest prefix with d_i = g_{i-1}; emit
+// d_1..d_a and g_a; KV length becomes pos + a + 1 (rows beyond it are stale
+// and rewritten before any read); the full model's max-probabilities of rows
+// 0..a join the C_trace window; g_a is the next pending token.
+__global__ void k_accept(Dims D, Bufs B, cudaGraphConditionalHandle gen_while) {
+  Ctl* c = B.ctl;
+  ssd_round_trace& r = c->cur;
+  const int k = c->k;
+  int a = 0;
+  while (a < k && c->tok[a + 1] == B.stats[a].argmax) ++a;
+  for (int i = 0; i <= k; ++i) {
+    r.verify_tok[i] = B.stats[i].argmax;
+    r.verify_margin[i] = B.stats[i].margin;
+    r.verify_pmax[i] = B.stats[i].pmax;
+  }
+  const int g = B.stats[a].argmax;
+  for (int i = 0; i < a; ++i) r.emitted[i] = c->tok[i + 1];
+  r.emitted[a] = g;
+  for (int i = 0; i <= a; ++i) {
+    if (c->n_out + i < D.max_seq) B.out_tok[c->n_out + i] = r.emitted[i];
+    trace_push(c, B.stats[i].pmax);
+  }
+  r.lstar = c->lstar;
+  r.k = k;
+  r.a = a;
+  r.n_emit = a + 1;
+  if (c->round_idx < D.max_seq) B.traces[c->round_idx] = r;
+  else atomicOr(&c->err, (int)kErrTraceFull);
+  c->n_out += a + 1;
+  c->pos += a + 1;
+  c->x = g;
+  c->round_idx += 1;
+  set_cond(gen_while, c->n_out < c->max_new ? 1u : 0u);
+}
+
+__global__ void k_begin_call(Bufs B, int max_new) {
+  Ctl* c = B.ctl;
+  c->max_new = max_new;
+  c->n_out = 0;
+  c->round_idx = 0;
+  c->err = 0;
+}
+
+__global__ void k_reset_sequence(Bufs B) {
+  Ctl* c = B.ctl;
+  c->pos = 0;
+  c->x = 0;
+  c->n_out = 0;
+  c->round_idx = 0;
+  c->trace_n = 0;
+  c->trace_head = 0;
+  c->err = 0;
+}
+
+__global__ void k_trace_push(Bufs B, int first_row, int n_rows) {
+  for (int i = 0; i < n_rows; ++i) trace_push(B.ctl, B.stats[first_row + i].pmax);
+}
+
+// Pending token = argmax of stats[row] (token < 0) or the given token.
+__global__ void k_set_pending(Bufs B, int row, int token, int pos) {
+  Ctl* c = B.ctl;
+  c->x = token >= 0 ? token : B.stats[row].argmax;
+  c->pos = pos;
+}
+
+__global__ void k_qnet_eval(Bufs B, int H, const float* __restrict__ states, int n,
+                            float* __restrict__ q) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const float* W1 = B.qparams;
+  const float* b1 = W1 + 3 * H;
+  const float* W2 = b1 + H;
+  const float* b2 = W2 + 2 * H;
+  const float s0 = states[3 * i], s1 = states[3 * i + 1], s2 = states[3 * i + 2];
+  float a0 = 0.f, a1 = 0.f;
+  for (int j = 0; j < H; ++j) {
+    float z = b1[j];
+    z = fmaf(W1[3 * j], s0, z);
+    z = fmaf(W1[3 * j + 1], s1, z);
+    z = fmaf(W1[3 * j + 2], s2, z);
+    const float r = fmaxf(z, 0.f);
+    a0 = fmaf(W2[j], r, a0);
+    a1 = fmaf(W2[H + j], r, a1);
+  }
+  q[2 * i] = a0 + b2[0];
+  q[2 * i + 1] = a1 + b2[1];
+}
+
+// Test fixture: seeded synthetic weights (synth.h), grid-stride.
+__global__ void k_synth_fill(void* dst, int dtype, uint64_t n, uint32_t seed, uint32_t tid,
+                             double sigma) {
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+    const float v = synth_weight_f32(seed, tid, i, sigma);
+    if (dtype == SSD_DTYPE_BF16)
+      static_cast<uint16_t*>(dst)[i] = synth_f32_to_bf16(v);
+    else
+      static_cast<float*>(dst)[i] = v;
+  }
+}
+
+template <typename T>
+__global__ void k_kv_to_f32(Dims D, Bufs B, int layer, int kind, int head, int p0, int n,
+                            float* out) {
+  const T* kv = static_cast<const T*>(B.kv) + (size_t)layer * 2 * D.Hkv * D.max_seq * D.hd +
+                ((size_t)(kind * D.Hkv + head) * D.max_seq + p0) * D.hd;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n * D.hd; i += gridDim.x * blockDim.x)
+    out[i] = Elem<T>::to_f(kv[i]);
+}
+
+// ---------------------------------------------------------------- launchers
+
+cudaError_t launch_embed(const Dims& D, const Bufs& B, int dtype, const void* embed, RowSel sel,
+                         bool big, cudaGraphConditionalHandle sw, cudaStream_t st) {
+  const int grid = big ? kMaxM : 1;
+  if (dtype == SSD_DTYPE_BF16)
+    k_embed<__nv_bfloat16><<<grid, 256, 0, st>>>(D, B, static_cast<const __nv_bfloat16*>(embed),
+                                                  sel, sw);
+  else
+    k_embed<float><<<grid, 256, 0, st>>>(D, B, static_cast<const float*>(embed), sel, sw);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_round_begin(const Dims& D, const Bufs& B, cudaGraphConditionalHandle draft_if,
+                               cudaStream_t st) {
+  k_round_begin<<<1, 1, 0, st>>>(D, B, draft_if);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decide(const Dims& D, const Bufs& B, int mode, int cand_idx, int is_last,
+                          int layer, cudaGraphConditionalHandle next_if,
+                          cudaGraphConditionalHandle draft_while, cudaStream_t st) {
+  k_decide<<<1, 256, 0, st>>>(D, B, mode, cand_idx, is_last, layer, next_if, draft_while);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_draft_begin(const Bufs& B, cudaGraphConditionalHandle draft_while,
+                               cudaStream_t st) {
+  k_draft_begin<<<1, 1, 0, st>>>(B, draft_while);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_accept(const Dims& D, const Bufs& B, cudaGraphConditionalHandle gen_while,
+                          cudaStream_t st) {
+  k_accept<<<1, 1, 0, st>>>(D, B, gen_while);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_begin_call(const Bufs& B, int max_new, cudaStream_t st) {
+  k_begin_call<<<1, 1, 0, st>>>(B, max_new);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_reset_sequence(const Bufs& B, cudaStream_t st) {
+  k_reset_sequence<<<1, 1, 0, st>>>(B);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_trace_push(const Bufs& B, int first_row, int n_rows, cudaStream_t st) {
+  k_trace_push<<<1, 1, 0, st>>>(B, first_row, n_rows);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_set_pending(const Bufs& B, int stats_row, int token, int pos, cudaStream_t st) {
+  k_set_pending<<<1, 1, 0, st>>>(B, stats_row, token, pos);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_qnet_eval(const Bufs& B, int hidden, const float* states, int n, float* q,
+                             cudaStream_t st) {
+  k_qnet_eval<<<(n + 127) / 128, 128, 0, st>>>(B, hidden, states, n, q);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_synth_fill(void* dst, int dtype, uint64_t n, uint32_t seed, uint32_t tid,
+                              double sigma, cudaStream_t st) {
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  k_synth_fill<<<sms * 8, 256, 0, st>>>(dst, dtype, n, seed, tid, sigma);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_kv_to_f32(const Dims& D, const Bufs& B, int dtype, int layer, int kind,
+                             int head, int p0, int n, float* out, cudaStream_t st) {
+  const int blocks = (n * D.hd + 255) / 256;
+  if (dtype == SSD_DTYPE_BF16)
+    k_kv_to_f32<__nv_bfloat16><<<blocks, 256, 0, st>>>(D, B, layer, kind, head, p0, n, out);
+  else
+    k_kv_to_f32<float><<<blocks, 256, 0, st>>>(D, B, layer, kind, head, p0, n, out);
+  return cudaGetLastError();
+}
+
+}  // namespace ssd

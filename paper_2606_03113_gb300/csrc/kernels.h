@@ -1,0 +1,55 @@
+// kernels.h -- host-side launchers of the engine's kernels (internal).
+#pragma once
+
+#include "common.cuh"
+
+namespace ssd {
+
+// Statistics partial of one block of vocabulary rows (exit head, first stage).
+struct HeadPart {
+  float mx;  // max logit (== tv[0] when the block has rows)
+  float S;   // sum exp(z - mx)
+  float T;   // sum exp(z - mx) (z - mx)
+  float tv[kTopK];
+  int32_t ti[kTopK];
+};
+
+constexpr int kHeadRowsPerBlock = 2 * kWarps;
+
+inline int head_blocks(int V) { return (V + kHeadRowsPerBlock - 1) / kHeadRowsPerBlock; }
+
+// big = true selects the kernels instantiated for up to kMaxM rows; false
+// the single-row ones.
+cudaError_t launch_embed(const Dims& D, const Bufs& B, int dtype, const void* embed, RowSel sel,
+                         bool big, cudaGraphConditionalHandle set_lstar_switch, cudaStream_t st);
+cudaError_t launch_layer(const Dims& D, const Bufs& B, int dtype, const LayerW& w, int layer,
+                         RowSel sel, bool big, cudaStream_t st);
+cudaError_t launch_head(const Dims& D, const Bufs& B, int dtype, const void* lm_head,
+                        const void* final_norm, int topk, bool write_logits, RowSel sel, bool big,
+                        cudaStream_t st);
+cudaError_t launch_round_begin(const Dims& D, const Bufs& B, cudaGraphConditionalHandle draft_if,
+                               cudaStream_t st);
+cudaError_t launch_decide(const Dims& D, const Bufs& B, int mode, int cand_idx, int is_last,
+                          int layer, cudaGraphConditionalHandle next_if,
+                          cudaGraphConditionalHandle draft_while, cudaStream_t st);
+cudaError_t launch_draft_begin(const Bufs& B, cudaGraphConditionalHandle draft_while,
+                               cudaStream_t st);
+cudaError_t launch_accept(const Dims& D, const Bufs& B, cudaGraphConditionalHandle gen_while,
+                          cudaStream_t st);
+cudaError_t launch_begin_call(const Bufs& B, int max_new, cudaStream_t st);
+cudaError_t launch_reset_sequence(const Bufs& B, cudaStream_t st);
+cudaError_t launch_trace_push(const Bufs& B, int first_row, int n_rows, cudaStream_t st);
+cudaError_t launch_set_pending(const Bufs& B, int stats_row, int token, int pos, cudaStream_t st);
+cudaError_t launch_qnet_eval(const Bufs& B, int hidden, const float* states, int n, float* q,
+                             cudaStream_t st);
+cudaError_t launch_gemv_plain(int dtype, const void* W, int rows, int cols, const float* x, int M,
+                              float* y, cudaStream_t st);
+cudaError_t launch_synth_fill(void* dst, int dtype, uint64_t n, uint32_t seed, uint32_t tid,
+                              double sigma, cudaStream_t st);
+cudaError_t launch_read_probe(const void* src, uint64_t bytes, uint32_t* sink, cudaStream_t st);
+cudaError_t launch_kv_to_f32(const Dims& D, const Bufs& B, int dtype, int layer, int kind,
+                             int head, int p0, int n, float* out, cudaStream_t st);
+
+enum DecideMode : int { kDecideWalk = 0, kDecideDraft = 1 };
+
+}  // namespace ssd

@@ -13,8 +13,9 @@ import threading
 
 import numpy as np
 
-from .workloads import (QNET_IN, QNET_OUT, SEED_PROMPT, SEED_QNET, SEED_WEIGHTS, TOPK_CONF,
-                        TRACE_T, WORKLOADS, ModelShape, Workload, scaled_down)
+from .workloads import (LT_WDOWN, LT_WGU, LT_WO, LT_WQKV, QNET_IN, QNET_OUT, SEED_PROMPT,
+                        SEED_QNET, SEED_WEIGHTS, TID_EMBED, TID_LMHEAD, TOPK_CONF, TRACE_T,
+                        WORKLOADS, ModelShape, Workload, layer_tid, scaled_down)
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 BUILD_DIR = os.path.join(HERE, "_build")
@@ -103,4 +104,5 @@ def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
 __all__ = ["build", "lib", "philox4x32_10", "prompt_ids", "qnet_hidden_params", "weights_f32",
            "weights_bf16_bits", "bf16_bits_to_f32", "WORKLOADS", "ModelShape", "Workload",
            "scaled_down", "SEED_WEIGHTS", "SEED_PROMPT", "SEED_QNET", "TRACE_T", "TOPK_CONF",
-           "QNET_IN", "QNET_OUT", "HEADER"]
+           "QNET_IN", "QNET_OUT", "HEADER", "TID_EMBED", "TID_LMHEAD", "layer_tid",
+           "LT_WQKV", "LT_WO", "LT_WGU", "LT_WDOWN"]

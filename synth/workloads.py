@@ -21,6 +21,17 @@ SEED_WEIGHTS = 0
 SEED_PROMPT = 1
 SEED_QNET = 2
 
+# tensor ids of synth.h
+TID_EMBED = 1
+TID_LMHEAD = 2
+TID_LAYER_BASE = 16
+LT_WQKV, LT_WO, LT_WGU, LT_WDOWN = 0, 1, 2, 3
+
+
+def layer_tid(layer: int, which: int) -> int:
+    return TID_LAYER_BASE + 4 * layer + which
+
+
 TRACE_T = 20  # C_trace window (§3.1.1, T = 20)
 TOPK_CONF = 5  # token confidence C_k uses the top-5 probabilities (§3.1.1, k = 5)
 QNET_IN = 3  # state s = (C_5, H, C_trace)
