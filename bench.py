@@ -1,0 +1,379 @@
+"""Batch-1 decode throughput of self-speculative decoding with the LEDE policy
+on a synthetic Llama-2-7B-shaped decoder (bf16, prompt 512, 256 new tokens),
+beside plain GPU autoregressive decoding and static (l, k) speculation on the
+same kernels.
+
+One step = one generation of the workload's new tokens through the whole hot
+path (walk, drafting, verification, acceptance, rollback), timed with CUDA
+events on the engine's stream after an untimed prefill.  Weights (13.5 GB)
+are larger than L2, so no flush is needed between steps.
+
+Prints one JSON line.  --impl reference times the CPU oracle instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+REPO = os.path.dirname(os.path.abspath(__file__))
+if REPO not in sys.path:
+    sys.path.insert(0, REPO)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+from synth.workloads import WORKLOADS  # noqa: E402
+
+METRIC = "batch-1 decode tokens/sec and % of HBM-bandwidth roofline vs GPU AR/static"
+CLOCK_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+def measured_peaks() -> dict:
+    p = os.path.join(REPO, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(hbm_gbs=float(d["hbm_gbs"]), src="measured")
+    return dict(hbm_gbs=6800.0, src="fallback")
+
+
+# --------------------------------------------------------------- bytes model
+
+def round_bytes(w, tr: dict) -> float:
+    """HBM bytes the method must read in one round: for each visited
+    candidate the LM head, the layers up to l* once for the pending token,
+    (k - 1) further drafts through l* layers + head, and the full model +
+    head for verification; KV reads of every layer pass at its context."""
+    s = w.shape
+    Wl, head = s.layer_weight_bytes(), s.lm_head_bytes()
+    kvpl = s.kv_bytes_per_pos_layer()
+    L, pos = s.n_layers, tr["pos"]
+    b = 0.0
+    if tr["kcap"] > 0:
+        l_star, k = tr["lstar"], tr["k"]
+        b += len(tr["visited"]) * head + l_star * (Wl + kvpl * (pos + 1))
+        for i in range(1, k):
+            b += l_star * (Wl + kvpl * (pos + i + 1)) + head
+    k = tr["k"]
+    b += L * (Wl + kvpl * (pos + k + 1)) + head
+    return b
+
+
+def kernels_in_round(w, tr: dict) -> int:
+    from paper_2606_03113_gb300.runtime import kernels_per_round
+    return kernels_per_round(tr, w.shape.n_layers, 0)
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    def __init__(self, device_index: int):
+        self.idx = device_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.idx}", f"--query-gpu={CLOCK_FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self) -> dict:
+        rows = []
+        if self.path and os.path.exists(self.path):
+            for line in open(self.path):
+                f = [x.strip() for x in line.split(",")]
+                if len(f) >= 9:
+                    rows.append(f)
+            os.unlink(self.path)
+        if not rows:
+            return dict(sm_mhz=None, sm_max_mhz=None, reasons=["unavailable"], samples=0)
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        reasons = set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in rows:
+            for name, v in zip(names, r[5:9]):
+                if v.lower() == "active":
+                    reasons.add(name)
+        return dict(sm_mhz=statistics.median(sm) if sm else None,
+                    sm_max_mhz=max(mx) if mx else None, reasons=sorted(reasons),
+                    samples=len(rows))
+
+
+# --------------------------------------------------------------- oracle arm
+
+def oracle_sample(w, n_prompt: int, n_new: int, policy: str, om=None) -> dict:
+    """Times the CPU oracle (as it stands) on a bounded sample of the
+    workload: prefill of the first n_prompt prompt tokens, then n_new decoded
+    tokens; the decode rate is the reported number."""
+    import oracle
+    t0 = time.perf_counter()
+    om = om or oracle.Model(w.shape)
+    t_model = time.perf_counter() - t0
+    ids = synth.prompt_ids(n_prompt, w.shape.vocab)
+    s = om.session(n_prompt + n_new + w.kmax + 2)
+    s.prefill(ids)
+    if policy == "ar":
+        P = oracle.make_policy(oracle.POLICY_AR)
+    else:
+        P = oracle.make_policy(oracle.POLICY_LEDE, w.candidates, kmax=w.kmax,
+                               q_params=synth.qnet_hidden_params(3, w.qnet_hidden),
+                               q_hidden=w.qnet_hidden)
+    t1 = time.perf_counter()
+    out, logs = s.generate(P, n_new)
+    dt = time.perf_counter() - t1
+    return dict(value=n_new / dt, seconds=dt, model_seconds=t_model, cores=oracle.num_threads(),
+                model=om,
+                sample=f"{w.name}-shaped oracle (fp64), {policy} policy: prefill of the first "
+                       f"{n_prompt} prompt tokens (untimed), then {n_new} decoded tokens timed")
+
+
+def run_reference(args, w, rank: int, world: int):
+    if rank != 0:
+        return
+    steps = []
+    samples = None
+    om = None
+    for i in range(args.warmup + args.steps):
+        r = oracle_sample(w, args.ref_prompt, args.ref_new, args.policy, om)
+        om = r["model"]
+        if i >= args.warmup:
+            steps.append(r)
+        samples = r
+    tok = args.ref_new * len(steps)
+    sec = sum(r["seconds"] for r in steps)
+    value = tok / sec
+    line = dict(metric=METRIC, value=value, unit="tokens/s", n_gpus=world, steps=args.steps,
+                warmup=args.warmup, ms_per_step=1e3 * sec / len(steps), higher_is_better=True,
+                scaling="weak", vs_baseline=None, dtype="f64", data="synthetic", impl="reference",
+                config=dict(workload=f"{w.name}-shaped decoder, batch 1, {args.policy} policy",
+                            sample=samples["sample"]),
+                cpu_baseline=dict(value=value, unit="tokens/s", cores=samples["cores"],
+                                  kind="oracle", sample=samples["sample"]),
+                e2e=dict(value=value, unit="tokens/s", h2d_bytes_per_step=0,
+                         d2h_bytes_per_step=0))
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------ GPU arm
+
+def time_generate(eng, ids, n_new, dist_barrier) -> tuple:
+    import torch
+    eng.prefill(ids)
+    dist_barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(eng.stream)
+    eng.generate_async(n_new)
+    e1.record(eng.stream)
+    nr, ne, tr = eng.generate_result(traces=True, cap=n_new)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1), ne, tr
+
+
+KERNEL_NAMES = {0: "k_qkv", 1: "k_attn+k_attn_combine", 2: "k_resid(wo)", 3: "k_gate_up",
+                4: "k_resid(w_down)", 5: "k_head"}
+
+
+def kernel_roofline(eng, w, peak: float, pos0: int, iters: int = 3) -> dict:
+    """Live CUDA-event timing (on the engine's stream, where the kernels are
+    launched) of each hot-path kernel of a single-row pass, one launch per
+    layer over all layers, so a launch never finds its weights in L2.  Bytes
+    are the algorithmic ones: the weight matrix (plus norm weights) of the
+    launch; attention counts its K/V reads at context pos0."""
+    import torch
+    s = w.shape
+    L = s.n_layers
+    elt = s.elt_bytes
+    qd = s.n_heads * s.head_dim
+    byts = {0: s.qkv_rows * s.d_model * elt, 1: s.kv_bytes_per_pos_layer() * (pos0 + 1),
+            2: s.d_model * qd * elt, 3: 2 * s.ffn_dim * s.d_model * elt,
+            4: s.d_model * s.ffn_dim * elt, 5: s.vocab * s.d_model * elt}
+    out = {}
+    st = eng.stream
+    for kern in (0, 1, 2, 3, 4, 5):
+        layers = [0] if kern == 5 else list(range(L))
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        for rep in range(iters + 1):
+            e0.record(st)
+            for l in layers:
+                eng.op_layer(kern, l, 1, pos0)
+            e1.record(st)
+        torch.cuda.synchronize()
+        us = e0.elapsed_time(e1) * 1e3 / len(layers)
+        b = byts[kern]
+        out[KERNEL_NAMES[kern]] = dict(us=us, bytes=b, launches_per_forward=len(layers),
+                                       gbs=b / us / 1e3, frac=b / us / 1e3 / peak)
+    return out
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama2-7b", choices=sorted(WORKLOADS))
+    ap.add_argument("--policy", default="lede", choices=["lede", "ar", "static"])
+    ap.add_argument("--gen", type=int, default=0, help="new tokens per step (default: workload)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-compare", action="store_true", help="skip the AR / static lines")
+    ap.add_argument("--ref-prompt", type=int, default=16)
+    ap.add_argument("--ref-new", type=int, default=4)
+    args = ap.parse_args()
+
+    w = WORKLOADS[args.workload]
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        run_reference(args, w, rank, world)
+        return
+
+    import torch
+    import torch.distributed as dist
+    if world > 1:
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    from paper_2606_03113_gb300.runtime import DeviceModel, Engine
+    peaks = measured_peaks()
+    peak = peaks["hbm_gbs"]
+    n_new = args.gen or w.gen_len
+    model = DeviceModel(w.shape, f"cuda:{local}")
+    stream = torch.cuda.Stream(device=local)
+    eng = Engine(model, w.max_seq, stream=stream)
+    ids = synth.prompt_ids(w.prompt_len, w.shape.vocab)
+
+    def set_policy(kind, l=0, k=0):
+        if kind == "ar":
+            eng.set_ar()
+        elif kind == "static":
+            eng.set_static(l, k, kmax=w.kmax)
+        else:
+            eng.set_lede(w, synth.qnet_hidden_params(3, w.qnet_hidden))
+
+    L = w.shape.n_layers
+    static_lk = (max(1, L // 4), 4)  # the LayerSkip-style default (E = L/4, d = 4)
+    set_policy(args.policy, *static_lk)
+    for _ in range(args.warmup):
+        time_generate(eng, ids, n_new, barrier)
+    results = []
+    with ClockSampler(local) as clk:
+        for _ in range(args.steps):
+            results.append(time_generate(eng, ids, n_new, barrier))
+    clocks = clk.summary()
+    ms = [r[0] for r in results]
+    toks = [r[1] for r in results]
+    local_ms = sum(ms)
+    if world > 1:
+        t = torch.tensor([local_ms, float(sum(toks))], device=f"cuda:{local}")
+        mx = t.clone()
+        dist.all_reduce(mx[:1], op=dist.ReduceOp.MAX)
+        dist.all_reduce(t[1:], op=dist.ReduceOp.SUM)
+        total_ms, total_tok = float(mx[0]), float(t[1])
+    else:
+        total_ms, total_tok = local_ms, float(sum(toks))
+    value = total_tok / (total_ms / 1e3)
+    traces = results[-1][2]
+    bytes_step = sum(round_bytes(w, tr) for tr in traces)
+    step_gbs = bytes_step / (results[-1][0] / 1e3) / 1e9
+    launches = sum(sum(kernels_in_round(w, tr) for tr in r[2]) for r in results)
+    acc_k = sum(tr["k"] for tr in traces)
+    policy_stats = dict(rounds=len(traces), E=float(np.mean([t["lstar"] for t in traces if t["kcap"] > 0]
+                                                            or [0])),
+                        d=acc_k / max(1, sum(1 for t in traces if t["kcap"] > 0)),
+                        acc_rate=sum(t["a"] for t in traces) / max(1, acc_k),
+                        tokens_per_round=n_new / max(1, len(traces)),
+                        gb_per_token=bytes_step / n_new / 1e9)
+
+    # e2e through the public API with host buffers: prompt in, tokens out
+    from paper_2606_03113_gb300 import ssd as S
+    t0 = time.perf_counter()
+    S.ssd_prefill(eng.ctx, ids)
+    out, _, _ = S.ssd_generate(eng.ctx, n_new)
+    e2e_s = time.perf_counter() - t0
+    e2e = dict(value=n_new / e2e_s, unit="tokens/s", h2d_bytes_per_step=int(ids.nbytes),
+               d2h_bytes_per_step=int(out.nbytes),
+               note="ssd_prefill (host prompt) + ssd_generate (host tokens), wall clock")
+
+    roof = kernel_roofline(eng, w, peak, pos0=w.prompt_len + n_new // 2)
+    dom = max(roof.items(), key=lambda kv: kv[1]["us"] * kv[1]["launches_per_forward"])
+    roofline = dict(bound="hbm", achieved=dom[1]["gbs"], peak=peak, unit="GB/s",
+                    frac=dom[1]["gbs"] / peak, traffic=None,
+                    kernel=f"{dom[0]} single-row ({dom[1]['bytes'] / 1e6:.1f} MB per launch)",
+                    peak_source=f"{peaks['src']} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
+                    kernels=roof,
+                    decode_step=dict(achieved=step_gbs, frac=step_gbs / peak,
+                                     what="weight + KV bytes the round structure must read / step time"))
+
+    compare = {}
+    if not args.no_compare and args.policy == "lede":
+        for name, kind, lk in (("ar", "ar", (0, 0)), ("static_layerskip", "static", static_lk),
+                               ("static_l16_k4", "static", (L // 2, 4)),
+                               ("static_l24_k2", "static", (3 * L // 4, 2))):
+            set_policy(kind, *lk)
+            time_generate(eng, ids, n_new, barrier)
+            r = time_generate(eng, ids, n_new, barrier)
+            tr = r[2]
+            compare[name] = dict(tok_s=r[1] / (r[0] / 1e3), l=lk[0], k=lk[1],
+                                 acc_rate=sum(t["a"] for t in tr) / max(1, sum(t["k"] for t in tr)),
+                                 gb_per_token=sum(round_bytes(w, t) for t in tr) / r[1] / 1e9)
+        ar_bytes = L * w.shape.layer_weight_bytes() + w.shape.lm_head_bytes()
+        compare["ar_roofline_tok_s"] = peak * 1e9 / ar_bytes
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline and world == 1:
+        r = oracle_sample(w, args.ref_prompt, args.ref_new, args.policy)
+        cpu = dict(value=r["value"], unit="tokens/s", cores=r["cores"], kind="oracle",
+                   sample=r["sample"])
+
+    line = dict(metric=METRIC, value=value, unit="tokens/s", n_gpus=world, steps=args.steps,
+                warmup=args.warmup, ms_per_step=total_ms / args.steps, higher_is_better=True,
+                scaling="weak", vs_baseline=None, dtype="bf16", data="synthetic",
+                config=dict(workload=f"{w.name}-shaped decoder (random-init bf16), batch 1, "
+                                     f"prompt {w.prompt_len}, {n_new} new tokens per step, "
+                                     f"{args.policy} policy"
+                                     + (" (seeded Q-network)" if args.policy == "lede" else ""),
+                            l2="inputs larger than L2 (13.5 GB of weights streamed per pass)",
+                            parallelism=f"replicas x{world}" if world > 1 else "single GPU"),
+                roofline=roofline, cpu_baseline=cpu, e2e=e2e, gpu_launches=launches,
+                clocks=clocks, policy_stats=policy_stats, compare=compare)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    eng.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

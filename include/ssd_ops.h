@@ -57,6 +57,17 @@ ssd_status ssd_read_state(ssd_ctx* ctx, int32_t* x, int32_t* pos, float* trace, 
 ssd_status ssd_op_gemv(ssd_ctx* ctx, int32_t which, int32_t layer, int32_t M, const float* x_dev,
                        float* y_dev, void* stream);
 
+/* One launch of one hot-path kernel of layer `layer` exactly as the round
+ * graphs launch it, on M rows at positions pos0..pos0+M-1 of the context's
+ * own buffers: kernel = 0 QKV (+RoPE, KV append), 1 attention (split-K and
+ * combine), 2 O projection (+residual), 3 gate/up (+RMSNorm, SwiGLU),
+ * 4 down projection (+residual), 5 exit head (final RMSNorm, LM head,
+ * statistics; layer ignored).  It overwrites the activations and the KV rows
+ * at those positions: for timing and profiling, not inside a generation.
+ * Needs pos0 + M <= max_seq.  Enqueued on `stream` (NULL = the context's). */
+ssd_status ssd_op_layer(ssd_ctx* ctx, int32_t kernel, int32_t layer, int32_t M, int32_t pos0,
+                        void* stream);
+
 /* Test fixture: fills dst (device, n elements of dtype) with the seeded
  * synthetic weights of tensor `tid` (see synth/synth.h): element i is
  * synth_weight_f32(seed, tid, i, sigma), rounded to bf16 for SSD_DTYPE_BF16.

@@ -775,6 +775,24 @@ ssd_status ssd_op_gemv(ssd_ctx* x, int32_t which, int32_t layer, int32_t M, cons
   return SSD_OK;
 }
 
+ssd_status ssd_op_layer(ssd_ctx* x, int32_t kernel, int32_t layer, int32_t M, int32_t pos0,
+                        void* stream) {
+  if (!x) return fail(nullptr, SSD_ERR_INVALID_ARG, "ctx is NULL");
+  if (M < 1 || M > kMaxM || pos0 < 0 || pos0 + M > x->cfg.max_seq)
+    return fail(x, SSD_ERR_INVALID_ARG, "M must be in 1..17 with pos0 + M <= max_seq");
+  if (kernel < 0 || kernel > 5 || (kernel < 5 && (layer < 0 || layer >= x->cfg.n_layers)))
+    return fail(x, SSD_ERR_INVALID_ARG, "kernel must be 0..5 and layer in range");
+  cudaStream_t st = stream ? static_cast<cudaStream_t>(stream) : x->stream;
+  const RowSel sel = rows_explicit(pos0, M, x->B.pre_tok);
+  const bool big = M > 1;
+  if (kernel == 5)
+    CK(x, enqueue_head(x, sel, big, x->topk, false, st));
+  else
+    CK(x, launch_layer_part(x->D, x->B, x->cfg.dtype, x->layers[kernel == 5 ? 0 : layer], layer,
+                            kernel, sel, big, st));
+  return SSD_OK;
+}
+
 ssd_status ssd_synth_fill(void* dst, int32_t dtype, uint64_t n, uint32_t seed, uint32_t tid,
                           double sigma, void* stream) {
   if (!dst || (dtype != SSD_DTYPE_F32 && dtype != SSD_DTYPE_BF16))

@@ -457,6 +457,10 @@ __global__ void k_read_probe(const uint4* __restrict__ src, uint64_t n16, uint32
 
 // -------------------------------------------------------------- launchers
 
+// Attention launchers live in attention.cu.
+cudaError_t launch_attention(const Dims& D, const Bufs& B, int dtype, int layer, RowSel sel,
+                             bool big, cudaStream_t st);
+
 template <typename T, int MM>
 static cudaError_t layer_t(const Dims& D, const Bufs& B, const LayerW& w, int layer, RowSel sel,
                            cudaStream_t st);
@@ -479,31 +483,53 @@ cudaError_t launch_head(const Dims& D, const Bufs& B, int dtype, const void* lm_
              : head_t<float, 1>(D, B, lm_head, final_norm, topk, write_logits, sel, st);
 }
 
-// Attention launchers live in attention.cu.
-cudaError_t launch_attention(const Dims& D, const Bufs& B, int dtype, int layer, RowSel sel,
-                             bool big, cudaStream_t st);
+template <typename T, int MM>
+static cudaError_t part_t(const Dims& D, const Bufs& B, const LayerW& w, int layer, int part,
+                          RowSel sel, cudaStream_t st) {
+  const int threads = kWarps * 32;
+  switch (part) {
+    case 0: {
+      const int qkv_units = (D.Hq + 2 * D.Hkv) * D.hd / 2;
+      k_qkv<T, MM><<<(qkv_units + kWarps - 1) / kWarps, threads, 0, st>>>(D, B, w, layer, sel);
+      break;
+    }
+    case 1:
+      return launch_attention(D, B, std::is_same<T, float>::value ? SSD_DTYPE_F32 : SSD_DTYPE_BF16,
+                              layer, sel, MM > 1, st);
+    case 2:
+      k_resid<T, MM><<<D.res_blocks, threads, 0, st>>>(D, B, static_cast<const T*>(w.wo), D.qd,
+                                                       B.attn_out, 1, sel);
+      break;
+    case 3:
+      k_gate_up<T, MM><<<(D.F + kWarps - 1) / kWarps, threads, 0, st>>>(D, B, w, sel);
+      break;
+    case 4:
+      k_resid<T, MM><<<D.res_blocks, threads, 0, st>>>(D, B, static_cast<const T*>(w.wdown), D.F,
+                                                       B.act, 0, sel);
+      break;
+    default:
+      return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
 
 template <typename T, int MM>
 static cudaError_t layer_t(const Dims& D, const Bufs& B, const LayerW& w, int layer, RowSel sel,
                            cudaStream_t st) {
-  const int threads = kWarps * 32;
-  const int qkv_units = (D.Hq + 2 * D.Hkv) * D.hd / 2;
-  k_qkv<T, MM><<<(qkv_units + kWarps - 1) / kWarps, threads, 0, st>>>(D, B, w, layer, sel);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  e = launch_attention(D, B, std::is_same<T, float>::value ? SSD_DTYPE_F32 : SSD_DTYPE_BF16, layer,
-                       sel, MM > 1, st);
-  if (e != cudaSuccess) return e;
-  k_resid<T, MM><<<D.res_blocks, threads, 0, st>>>(D, B, static_cast<const T*>(w.wo), D.qd,
-                                                   B.attn_out, 1, sel);
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  k_gate_up<T, MM><<<(D.F + kWarps - 1) / kWarps, threads, 0, st>>>(D, B, w, sel);
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  k_resid<T, MM><<<D.res_blocks, threads, 0, st>>>(D, B, static_cast<const T*>(w.wdown), D.F,
-                                                   B.act, 0, sel);
-  return cudaGetLastError();
+  for (int part = 0; part < kLayerKernels - 1; ++part) {
+    cudaError_t e = part_t<T, MM>(D, B, w, layer, part, sel, st);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t launch_layer_part(const Dims& D, const Bufs& B, int dtype, const LayerW& w, int layer,
+                              int part, RowSel sel, bool big, cudaStream_t st) {
+  if (dtype == SSD_DTYPE_BF16)
+    return big ? part_t<__nv_bfloat16, kMaxM>(D, B, w, layer, part, sel, st)
+               : part_t<__nv_bfloat16, 1>(D, B, w, layer, part, sel, st);
+  return big ? part_t<float, kMaxM>(D, B, w, layer, part, sel, st)
+             : part_t<float, 1>(D, B, w, layer, part, sel, st);
 }
 
 cudaError_t launch_layer(const Dims& D, const Bufs& B, int dtype, const LayerW& w, int layer,

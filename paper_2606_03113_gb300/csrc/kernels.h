@@ -24,6 +24,9 @@ cudaError_t launch_embed(const Dims& D, const Bufs& B, int dtype, const void* em
                          bool big, cudaGraphConditionalHandle set_lstar_switch, cudaStream_t st);
 cudaError_t launch_layer(const Dims& D, const Bufs& B, int dtype, const LayerW& w, int layer,
                          RowSel sel, bool big, cudaStream_t st);
+// One kernel of a layer (0 qkv, 1 attention + combine, 2 o, 3 gate/up, 4 down).
+cudaError_t launch_layer_part(const Dims& D, const Bufs& B, int dtype, const LayerW& w, int layer,
+                              int part, RowSel sel, bool big, cudaStream_t st);
 cudaError_t launch_head(const Dims& D, const Bufs& B, int dtype, const void* lm_head,
                         const void* final_norm, int topk, bool write_logits, RowSel sel, bool big,
                         cudaStream_t st);

@@ -165,6 +165,10 @@ class Engine:
         st = (stream or self.stream).cuda_stream
         S.ssd_op_gemv(self.ctx, which, layer, M, x.data_ptr(), y.data_ptr(), st)
 
+    def op_layer(self, kernel: int, layer: int, M: int, pos0: int, stream=None):
+        st = (stream or self.stream).cuda_stream
+        S.ssd_op_layer(self.ctx, kernel, layer, M, pos0, st)
+
     def close(self):
         if getattr(self, "ctx", None):
             S.ssd_destroy(self.ctx)

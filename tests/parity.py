@@ -3,13 +3,14 @@
 Generation parity follows a segment-and-resync protocol.  The oracle
 generates the whole sequence once, logging every decision with its margin
 (token decisions: top-1 minus top-2 logit; Q decisions: |Q_exit - Q_continue|).
-The GPU replays it round by round from the same state.  A round whose
-decisions all have margins above the tolerance must match exactly (walk,
-exit layer, drafts, verification tokens, acceptance count, emitted tokens,
-Q actions; Q values within q_val_tol).  A round with a near-tie is not
-compared: both sides then restart from the oracle's emitted sequence
-(ssd_resume), which reproduces the oracle's state exactly (KV, trace window,
-pending token).
+The GPU replays it round by round from the same state.  Within a round the
+decisions are compared in the order they are taken, up to the first one the
+oracle takes with a margin at or below the tolerance: Q actions (values within
+q_val_tol), drafts, verification tokens, and the walk's exit layer once its
+decisions are all compared.  A round without a near-tie must match entirely
+(drafts, acceptance count, emitted tokens).  After a round with a near-tie
+the GPU restarts from the oracle's emitted sequence (ssd_resume), which
+reproduces the oracle's state (KV, trace window, pending token).
 """
 from __future__ import annotations
 
@@ -45,11 +46,58 @@ def set_gpu_policy(eng, kind: str, w, qp=None, l=0, k=0, kmax=None, cand=None):
         eng.set_lede(w, qp, kmax=kmax, cand=cand)
 
 
-def round_is_clear(lg: dict, tol_tok: float, tol_q: float) -> bool:
-    margins = list(lg["draft_margin"]) + list(lg["verify_margin"])
-    if margins and min(margins) <= tol_tok:
-        return False
-    return all(abs(q1 - q0) > tol_q for q0, q1 in lg["q_val"])
+def decisions(lg: dict, lede: bool) -> list:
+    """The round's decisions in the order they are taken: the walk's Q
+    decisions, d_1, then each further draft followed by the Q decision after
+    it, then the verification tokens g_0..g_k.  Each entry is
+    (kind, index, margin)."""
+    out = []
+    nv = len(lg["visited"]) if lede else 0
+    for i in range(nv):
+        q0, q1 = lg["q_val"][i]
+        out.append(("q", i, abs(q1 - q0)))
+    k = lg["k"]
+    for i in range(k):
+        out.append(("d", i, lg["draft_margin"][i]))
+        if lede and i >= 1:
+            q0, q1 = lg["q_val"][nv + i - 1]
+            out.append(("q", nv + i - 1, abs(q1 - q0)))
+    for i in range(k + 1):
+        out.append(("v", i, lg["verify_margin"][i]))
+    return out
+
+
+def compare_round(g: dict, lg: dict, lede: bool, tol_tok: float, tol_q: float,
+                  q_val_tol: float):
+    """Compares the GPU round g with the oracle round lg decision by decision
+    up to the first decision the oracle takes with a margin at or below the
+    tolerance.  Returns (compared, total, clear, max Q-value error)."""
+    ctx = f"round at pos {lg['pos']}: gpu {g} oracle {lg}"
+    assert g["pos"] == lg["pos"] and g["x"] == lg["x"] and g["kcap"] == lg["kcap"], ctx
+    ds = decisions(lg, lede)
+    n = 0
+    q_err = 0.0
+    for kind, i, margin in ds:
+        tol = tol_q if kind == "q" else tol_tok
+        if margin <= tol:
+            break
+        if kind == "q":
+            assert g["q_action"][i] == lg["q_action"][i], ("q", i, ctx)
+            q_err = max(q_err, *(abs(a - b) for a, b in zip(g["q_val"][i], lg["q_val"][i])))
+            assert q_err <= q_val_tol, (q_err, ctx)
+        elif kind == "d":
+            assert g["drafts"][i] == lg["drafts"][i], ("d", i, ctx)
+        else:
+            assert g["verify_tok"][i] == lg["verify_tok"][i], ("v", i, ctx)
+        n += 1
+    clear = n == len(ds)
+    walk_done = (not lede) or n >= len(lg["visited"])
+    if walk_done and lg["kcap"] > 0:
+        assert g["visited"] == lg["visited"] and g["lstar"] == lg["lstar"], ctx
+    if clear:
+        for key in ("k", "a", "emitted", "q_action"):
+            assert g[key] == lg[key], (key, ctx)
+    return n, len(ds), clear, q_err
 
 
 def first_token_margin(om, ids) -> float:
@@ -61,7 +109,7 @@ def first_token_margin(om, ids) -> float:
 
 def generation_parity(eng, om, w, ids, kind: str, n_new: int, tol_tok: float, tol_q: float,
                       q_val_tol: float, qp=None, l=0, k=0, kmax=None, cand=None) -> dict:
-    """Returns counts of compared / skipped rounds; asserts on every compared one."""
+    """Returns decision counts; asserts on every compared decision."""
     P = oracle_policy(kind, w, qp, l, k, kmax, cand)
     s = om.session(eng.max_seq)
     ofirst = s.prefill(ids)
@@ -72,32 +120,26 @@ def generation_parity(eng, om, w, ids, kind: str, n_new: int, tol_tok: float, to
     if gfirst != ofirst:
         assert first_token_margin(om, ids) <= tol_tok, (gfirst, ofirst)
         eng.resume(seq)
-    compared = skipped = 0
+    compared = total = clear_rounds = 0
     q_err = 0.0
     done = 0
+    lede = kind == "lede"
     for lg in logs:
         cap = n_new - done
-        clear = round_is_clear(lg, tol_tok, tol_q)
-        if clear:
-            toks, info = eng.step(cap)
-            g = eng.traces(1)[0]
-            ctx = f"round at pos {lg['pos']}: gpu {g} oracle {lg}"
-            assert g["pos"] == lg["pos"] and g["x"] == lg["x"] and g["kcap"] == lg["kcap"], ctx
-            for key in ("visited", "lstar", "k", "a", "drafts", "verify_tok", "emitted", "q_action"):
-                assert g[key] == lg[key], (key, ctx)
-            assert list(toks) == lg["emitted"], ctx
-            for (a0, a1), (b0, b1) in zip(g["q_val"], lg["q_val"]):
-                q_err = max(q_err, abs(a0 - b0), abs(a1 - b1))
-            assert q_err <= q_val_tol, (q_err, ctx)
-            compared += 1
-        else:
-            skipped += 1
+        eng.step(cap)
+        g = eng.traces(1)[0]
+        n, t, clear, qe = compare_round(g, lg, lede, tol_tok, tol_q, q_val_tol)
+        compared += n
+        total += t
+        clear_rounds += int(clear)
+        q_err = max(q_err, qe)
         seq += lg["emitted"]
         done += lg["n_emit"]
         if not clear and done < n_new:
             eng.resume(seq)
     assert done == n_new and seq[len(ids):] == [ofirst] + list(otoks)
-    return dict(compared=compared, skipped=skipped, rounds=len(logs), q_err=q_err)
+    return dict(compared=compared, decisions=total, clear_rounds=clear_rounds, rounds=len(logs),
+                q_err=q_err)
 
 
 def rel_err(a, b) -> float:

@@ -143,12 +143,14 @@ def test_teacher_forced_logits_and_stats(name):
     eng.set_ar()
     eng.prefill(ids[:n0])
     sess = om.session(w.max_seq)
+    worst = 0.0
     for l_exit in sorted({1, max(1, s.n_layers // 2), s.n_layers}):
         for M in (1, 17):
             z, st = eng.forward_exit(ids[n0:n0 + M], n0, l_exit)
             h = sess.forward(ids[:n0 + M], 0, 0, l_exit)
             for i in range(M):
                 zr, sr = om.exit_head(h[n0 + i])
+                worst = max(worst, rel_err(z[i], zr))
                 assert rel_err(z[i], zr) < tol_logit, (l_exit, M, i, rel_err(z[i], zr))
                 g = st[i]
                 if sr["margin"] > tol_tok:
@@ -160,6 +162,7 @@ def test_teacher_forced_logits_and_stats(name):
                 gaps = np.diff(sr["top_logit"])
                 if np.all(np.abs(gaps) > tol_tok):
                     assert g["top_idx"][:5] == sr["top_idx"][:5]
+    print(name, "max relative logit error", worst)
 
 
 def test_qnet_values_on_oracle_states():
@@ -188,7 +191,12 @@ def test_generation_matches_oracle(name, kind):
     r = generation_parity(eng, om, w, prompt(w), kind, w.gen_len, tol_tok, tol_q, q_val_tol,
                           qp=qp, **kw)
     print(name, kind, r)
-    assert r["compared"] >= max(1, r["rounds"] // 4), r
+    # A near-tie (about one bf16 decision in seven on these random-init
+    # models) ends the comparison of its round, so only a share of all
+    # decisions is compared: every compared one must match, and the share
+    # must not be vacuous (far larger for fp32).
+    need = 0.5 if w.shape.dtype == "f32" else 0.1
+    assert r["compared"] >= need * r["decisions"] and r["compared"] >= min(20, r["decisions"]), r
 
 
 def test_lede_always_exit_policy_drafts_to_cap():
@@ -200,7 +208,7 @@ def test_lede_always_exit_policy_drafts_to_cap():
         qp = np.zeros(6 * H + 2, dtype=np.float32)
         qp[-2], qp[-1] = qc, qe
         r = generation_parity(eng, om, w, prompt(w), "lede", 24, *TOL["bf16"][:2], 1e-3, qp=qp)
-        assert r["compared"] >= 1
+        assert r["compared"] >= 0.1 * r["decisions"], r
         for t in eng.traces(64):
             if t["kcap"] > 0:
                 if qe > qc:
