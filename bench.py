@@ -198,12 +198,13 @@ KERNEL_NAMES = {0: "k_qkv", 1: "k_attn+k_attn_combine", 2: "k_resid(wo)", 3: "k_
                 4: "k_resid(w_down)", 5: "k_head"}
 
 
-def kernel_roofline(eng, w, peak: float, pos0: int, iters: int = 3) -> dict:
-    """Live CUDA-event timing (on the engine's stream, where the kernels are
-    launched) of each hot-path kernel of a single-row pass, one launch per
-    layer over all layers, so a launch never finds its weights in L2.  Bytes
-    are the algorithmic ones: the weight matrix (plus norm weights) of the
-    launch; attention counts its K/V reads at context pos0."""
+def kernel_roofline(eng, w, peak: float, pos0: int, iters: int = 5, graphs: bool = True) -> dict:
+    """Live CUDA-event timing, on the engine's stream where the kernels are
+    launched, of each hot-path kernel of a single-row pass: one launch per
+    layer over all layers (so a launch never finds its weights in L2),
+    replayed from a CUDA graph so host launch cost does not enter.  Bytes are
+    the algorithmic ones: the launch's weight matrix; attention counts its
+    K/V reads at context pos0."""
     import torch
     s = w.shape
     L = s.n_layers
@@ -215,18 +216,36 @@ def kernel_roofline(eng, w, peak: float, pos0: int, iters: int = 3) -> dict:
     out = {}
     st = eng.stream
     for kern in (0, 1, 2, 3, 4, 5):
-        layers = [0] if kern == 5 else list(range(L))
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        for rep in range(iters + 1):
-            e0.record(st)
+        layers = [0] * 8 if kern == 5 else list(range(L))
+
+        def run():
             for l in layers:
                 eng.op_layer(kern, l, 1, pos0)
+
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        run()
+        torch.cuda.synchronize()
+        if graphs:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=st):
+                run()
+            with torch.cuda.stream(st):  # replay() launches on the current stream
+                g.replay()
+                torch.cuda.synchronize()
+                e0.record(st)
+                for _ in range(iters):
+                    g.replay()
+                e1.record(st)
+        else:
+            e0.record(st)
+            for _ in range(iters):
+                run()
             e1.record(st)
         torch.cuda.synchronize()
-        us = e0.elapsed_time(e1) * 1e3 / len(layers)
+        us = e0.elapsed_time(e1) * 1e3 / (iters * len(layers))
         b = byts[kern]
-        out[KERNEL_NAMES[kern]] = dict(us=us, bytes=b, launches_per_forward=len(layers),
+        out[KERNEL_NAMES[kern]] = dict(us=us, bytes=b, launches_per_forward=1 if kern == 5 else L,
                                        gbs=b / us / 1e3, frac=b / us / 1e3 / peak)
     return out
 
@@ -244,9 +263,19 @@ def main():
     ap.add_argument("--no-compare", action="store_true", help="skip the AR / static lines")
     ap.add_argument("--ref-prompt", type=int, default=16)
     ap.add_argument("--ref-new", type=int, default=4)
+    ap.add_argument("--kernels-only", action="store_true",
+                    help="prefill, then launch each hot-path kernel eagerly over all layers "
+                         "(for per-kernel ncu captures) and print their timings")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="override the layer count (small cases for ncu --set full)")
     args = ap.parse_args()
 
     w = WORKLOADS[args.workload]
+    if args.layers:
+        from dataclasses import replace
+        w = replace(w, shape=replace(w.shape, n_layers=args.layers,
+                                     name=f"{w.shape.name}-{args.layers}l"),
+                    candidates=tuple(c for c in w.candidates if c < args.layers) or (1,))
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
@@ -283,6 +312,14 @@ def main():
             eng.set_lede(w, synth.qnet_hidden_params(3, w.qnet_hidden))
 
     L = w.shape.n_layers
+    if args.kernels_only:
+        eng.set_ar()
+        eng.prefill(ids)
+        roof = kernel_roofline(eng, w, peak, pos0=w.prompt_len, iters=2, graphs=False)
+        if rank == 0:
+            print(json.dumps(dict(kernels=roof, workload=w.name, peak=peak)), flush=True)
+        eng.close()
+        return
     static_lk = (max(1, L // 4), 4)  # the LayerSkip-style default (E = L/4, d = 4)
     set_policy(args.policy, *static_lk)
     for _ in range(args.warmup):

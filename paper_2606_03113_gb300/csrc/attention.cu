@@ -12,6 +12,7 @@
 #include <math.h>
 
 #include "kernels.h"
+#include "pipe.cuh"
 
 namespace ssd {
 
@@ -20,6 +21,8 @@ __global__ void __launch_bounds__(kWarps * 32) k_attn(Dims D, Bufs B, int layer,
   extern __shared__ float sm[];
   const int split = blockIdx.x, g = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  pdl_wait();
+  pdl_launch_dependents();
   int pos0, M;
   resolve_rows(B.ctl, sel, pos0, M);
   const int s0 = split * kAttnChunk;
@@ -100,6 +103,8 @@ __global__ void __launch_bounds__(kWarps * 32) k_attn(Dims D, Bufs B, int layer,
 template <int MM>
 __global__ void k_attn_combine(Dims D, Bufs B, RowSel sel) {
   const int qh = blockIdx.x, m = blockIdx.y;
+  pdl_wait();
+  pdl_launch_dependents();
   int pos0, M;
   resolve_rows(B.ctl, sel, pos0, M);
   if (m >= M) return;
@@ -135,11 +140,10 @@ static cudaError_t attn_t(const Dims& D, const Bufs& B, int layer, RowSel sel, c
                                          (int)smem);
     if (e != cudaSuccess) return e;
   }
-  k_attn<T, MM><<<grid, kWarps * 32, smem, st>>>(D, B, layer, sel);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_ex(k_attn<T, MM>, grid, dim3(kWarps * 32), smem, st, D, B, layer, sel);
   if (e != cudaSuccess) return e;
-  k_attn_combine<MM><<<dim3(D.Hq, MM), D.hd < 128 ? D.hd : 128, 0, st>>>(D, B, sel);
-  return cudaGetLastError();
+  return launch_ex(k_attn_combine<MM>, dim3(D.Hq, MM), dim3(D.hd < 128 ? D.hd : 128), 0, st, D, B,
+                   sel);
 }
 
 cudaError_t launch_attention(const Dims& D, const Bufs& B, int dtype, int layer, RowSel sel,

@@ -63,7 +63,8 @@ enum ErrBits : int32_t {
   kErrToken = 1,      // a token id outside [0, vocab)
   kErrCapacity = 2,   // KV capacity would be exceeded
   kErrControl = 4,    // inconsistent round state (l*, k)
-  kErrTraceFull = 8   // more rounds than trace records
+  kErrTraceFull = 8,  // more rounds than trace records
+  kErrTimeout = 16    // a pipeline wait gave up (see the streamed kernels)
 };
 
 __device__ __forceinline__ void resolve_rows(const Ctl* c, const RowSel& s, int& pos0, int& M) {
@@ -138,7 +139,7 @@ struct LayerW {
 
 // Shapes and buffers every kernel may need.
 struct Dims {
-  int32_t L, d, Hq, Hkv, hd, F, V, max_seq, qd, kvd, nsplit, res_blocks;
+  int32_t L, d, Hq, Hkv, hd, F, V, max_seq, qd, kvd, nsplit, num_sms, ss_tiles;
   float eps;
 };
 
@@ -146,15 +147,18 @@ struct Bufs {
   Ctl* ctl;
   float* h;          // [kMaxM][d] residual stream
   float* ss;         // [2][kMaxM] sum of squares of h rows: [0] after down/embed, [1] after O
-  float* ss_part;    // [2][kMaxM][res_blocks] per-block partials of ss
-  uint32_t* ss_counter;  // [2] block tickets of the residual kernels
+  float* ss_tile;    // [2][ss_tiles][kMaxM] per-tile partials of ss
+  uint32_t* ss_counter;  // [2] tile tickets of the residual kernels
+  float* gpart;      // [num_sms][2][32][kMaxM] partial tile sums of blocks sharing a tile
+  uint32_t* tile_counter;      // [max tiles] tickets of shared tiles
+  uint32_t* head_group_counter;  // [head groups] tickets of the exit-head merge
   float* xq;         // [kMaxM][qd] rotated queries
   float* attn_part;  // [kMaxM][Hq][nsplit][hd] unnormalised partial outputs
   float* attn_ml;    // [kMaxM][Hq][nsplit][2] partial (max, sum)
   float* attn_out;   // [kMaxM][qd]
   float* act;        // [kMaxM][F]
   float* logits;     // [kMaxM][V] (written only when requested)
-  void* head_part;   // [kMaxM][head blocks] partial statistics
+  void* head_part;   // [head tiles + head groups][kMaxM] statistics partials
   uint32_t* head_counter;
   RowStats* stats;   // [kMaxM]
   float2* rope;      // [max_seq][hd/2] (cos, sin)

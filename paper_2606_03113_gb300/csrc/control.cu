@@ -7,6 +7,7 @@
 
 #include "../../synth/synth.h"
 #include "kernels.h"
+#include "pipe.cuh"
 
 namespace ssd {
 
@@ -36,6 +37,8 @@ __device__ float trace_conf(const Ctl* c, int T) {
 template <typename T>
 __global__ void k_embed(Dims D, Bufs B, const T* __restrict__ emb, RowSel sel,
                         cudaGraphConditionalHandle sw) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ float red[32];
   Ctl* c = B.ctl;
   int pos0, M;
@@ -75,6 +78,8 @@ __global__ void k_embed(Dims D, Bufs B, const T* __restrict__ emb, RowSel sel,
 // Draft cap of the round: min(kmax, tokens still to emit - 1), the static
 // length for a static policy, and the KV capacity.
 __global__ void k_round_begin(Dims D, Bufs B, cudaGraphConditionalHandle draft_if) {
+  pdl_wait();
+  pdl_launch_dependents();
   Ctl* c = B.ctl;
   const DevPolicy& P = c->pol;
   const int remaining = c->max_new - c->n_out;
@@ -118,6 +123,8 @@ __global__ void k_round_begin(Dims D, Bufs B, cudaGraphConditionalHandle draft_i
 __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, int layer,
                          cudaGraphConditionalHandle next_if,
                          cudaGraphConditionalHandle draft_while) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ float s_state[3];
   __shared__ float red0[32], red1[32];
   Ctl* c = B.ctl;
@@ -210,6 +217,8 @@ __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, in
 }
 
 __global__ void k_draft_begin(Bufs B, cudaGraphConditionalHandle draft_while) {
+  pdl_wait();
+  pdl_launch_dependents();
   set_cond(draft_while, (unsigned)B.ctl->keep);
 }
 
@@ -219,6 +228,8 @@ __global__ void k_draft_begin(Bufs B, cudaGraphConditionalHandle draft_while) {
 // and rewritten before any read); the full model's max-probabilities of rows
 // 0..a join the C_trace window; g_a is the next pending token.
 __global__ void k_accept(Dims D, Bufs B, cudaGraphConditionalHandle gen_while) {
+  pdl_wait();
+  pdl_launch_dependents();
   Ctl* c = B.ctl;
   ssd_round_trace& r = c->cur;
   const int k = c->k;
@@ -250,6 +261,8 @@ __global__ void k_accept(Dims D, Bufs B, cudaGraphConditionalHandle gen_while) {
 }
 
 __global__ void k_begin_call(Bufs B, int max_new) {
+  pdl_wait();
+  pdl_launch_dependents();
   Ctl* c = B.ctl;
   c->max_new = max_new;
   c->n_out = 0;
@@ -258,6 +271,8 @@ __global__ void k_begin_call(Bufs B, int max_new) {
 }
 
 __global__ void k_reset_sequence(Bufs B) {
+  pdl_wait();
+  pdl_launch_dependents();
   Ctl* c = B.ctl;
   c->pos = 0;
   c->x = 0;
@@ -269,11 +284,15 @@ __global__ void k_reset_sequence(Bufs B) {
 }
 
 __global__ void k_trace_push(Bufs B, int first_row, int n_rows) {
+  pdl_wait();
+  pdl_launch_dependents();
   for (int i = 0; i < n_rows; ++i) trace_push(B.ctl, B.stats[first_row + i].pmax);
 }
 
 // Pending token = argmax of stats[row] (token < 0) or the given token.
 __global__ void k_set_pending(Bufs B, int row, int token, int pos) {
+  pdl_wait();
+  pdl_launch_dependents();
   Ctl* c = B.ctl;
   c->x = token >= 0 ? token : B.stats[row].argmax;
   c->pos = pos;
@@ -281,6 +300,8 @@ __global__ void k_set_pending(Bufs B, int row, int token, int pos) {
 
 __global__ void k_qnet_eval(Bufs B, int H, const float* __restrict__ states, int n,
                             float* __restrict__ q) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   const float* W1 = B.qparams;
@@ -318,6 +339,8 @@ __global__ void k_synth_fill(void* dst, int dtype, uint64_t n, uint32_t seed, ui
 template <typename T>
 __global__ void k_kv_to_f32(Dims D, Bufs B, int layer, int kind, int head, int p0, int n,
                             float* out) {
+  pdl_wait();
+  pdl_launch_dependents();
   const T* kv = static_cast<const T*>(B.kv) + (size_t)layer * 2 * D.Hkv * D.max_seq * D.hd +
                 ((size_t)(kind * D.Hkv + head) * D.max_seq + p0) * D.hd;
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n * D.hd; i += gridDim.x * blockDim.x)
@@ -330,62 +353,53 @@ cudaError_t launch_embed(const Dims& D, const Bufs& B, int dtype, const void* em
                          bool big, cudaGraphConditionalHandle sw, cudaStream_t st) {
   const int grid = big ? kMaxM : 1;
   if (dtype == SSD_DTYPE_BF16)
-    k_embed<__nv_bfloat16><<<grid, 256, 0, st>>>(D, B, static_cast<const __nv_bfloat16*>(embed),
-                                                  sel, sw);
-  else
-    k_embed<float><<<grid, 256, 0, st>>>(D, B, static_cast<const float*>(embed), sel, sw);
-  return cudaGetLastError();
+      return launch_ex(k_embed<__nv_bfloat16>, dim3(grid), dim3(256), 0, st, D, B,
+                     static_cast<const __nv_bfloat16*>(embed), sel, sw);
+  return launch_ex(k_embed<float>, dim3(grid), dim3(256), 0, st, D, B,
+                   static_cast<const float*>(embed), sel, sw);
 }
 
 cudaError_t launch_round_begin(const Dims& D, const Bufs& B, cudaGraphConditionalHandle draft_if,
                                cudaStream_t st) {
-  k_round_begin<<<1, 1, 0, st>>>(D, B, draft_if);
-  return cudaGetLastError();
+  return launch_ex(k_round_begin, dim3(1), dim3(1), 0, st, D, B, draft_if);
 }
 
 cudaError_t launch_decide(const Dims& D, const Bufs& B, int mode, int cand_idx, int is_last,
                           int layer, cudaGraphConditionalHandle next_if,
                           cudaGraphConditionalHandle draft_while, cudaStream_t st) {
-  k_decide<<<1, 256, 0, st>>>(D, B, mode, cand_idx, is_last, layer, next_if, draft_while);
-  return cudaGetLastError();
+  return launch_ex(k_decide, dim3(1), dim3(256), 0, st, D, B, mode, cand_idx, is_last, layer,
+                   next_if, draft_while);
 }
 
 cudaError_t launch_draft_begin(const Bufs& B, cudaGraphConditionalHandle draft_while,
                                cudaStream_t st) {
-  k_draft_begin<<<1, 1, 0, st>>>(B, draft_while);
-  return cudaGetLastError();
+  return launch_ex(k_draft_begin, dim3(1), dim3(1), 0, st, B, draft_while);
 }
 
 cudaError_t launch_accept(const Dims& D, const Bufs& B, cudaGraphConditionalHandle gen_while,
                           cudaStream_t st) {
-  k_accept<<<1, 1, 0, st>>>(D, B, gen_while);
-  return cudaGetLastError();
+  return launch_ex(k_accept, dim3(1), dim3(1), 0, st, D, B, gen_while);
 }
 
 cudaError_t launch_begin_call(const Bufs& B, int max_new, cudaStream_t st) {
-  k_begin_call<<<1, 1, 0, st>>>(B, max_new);
-  return cudaGetLastError();
+  return launch_ex(k_begin_call, dim3(1), dim3(1), 0, st, B, max_new);
 }
 
 cudaError_t launch_reset_sequence(const Bufs& B, cudaStream_t st) {
-  k_reset_sequence<<<1, 1, 0, st>>>(B);
-  return cudaGetLastError();
+  return launch_ex(k_reset_sequence, dim3(1), dim3(1), 0, st, B);
 }
 
 cudaError_t launch_trace_push(const Bufs& B, int first_row, int n_rows, cudaStream_t st) {
-  k_trace_push<<<1, 1, 0, st>>>(B, first_row, n_rows);
-  return cudaGetLastError();
+  return launch_ex(k_trace_push, dim3(1), dim3(1), 0, st, B, first_row, n_rows);
 }
 
 cudaError_t launch_set_pending(const Bufs& B, int stats_row, int token, int pos, cudaStream_t st) {
-  k_set_pending<<<1, 1, 0, st>>>(B, stats_row, token, pos);
-  return cudaGetLastError();
+  return launch_ex(k_set_pending, dim3(1), dim3(1), 0, st, B, stats_row, token, pos);
 }
 
 cudaError_t launch_qnet_eval(const Bufs& B, int hidden, const float* states, int n, float* q,
                              cudaStream_t st) {
-  k_qnet_eval<<<(n + 127) / 128, 128, 0, st>>>(B, hidden, states, n, q);
-  return cudaGetLastError();
+  return launch_ex(k_qnet_eval, dim3((n + 127) / 128), dim3(128), 0, st, B, hidden, states, n, q);
 }
 
 cudaError_t launch_synth_fill(void* dst, int dtype, uint64_t n, uint32_t seed, uint32_t tid,
@@ -401,10 +415,10 @@ cudaError_t launch_kv_to_f32(const Dims& D, const Bufs& B, int dtype, int layer,
                              int head, int p0, int n, float* out, cudaStream_t st) {
   const int blocks = (n * D.hd + 255) / 256;
   if (dtype == SSD_DTYPE_BF16)
-    k_kv_to_f32<__nv_bfloat16><<<blocks, 256, 0, st>>>(D, B, layer, kind, head, p0, n, out);
-  else
-    k_kv_to_f32<float><<<blocks, 256, 0, st>>>(D, B, layer, kind, head, p0, n, out);
-  return cudaGetLastError();
+    return launch_ex(k_kv_to_f32<__nv_bfloat16>, dim3(blocks), dim3(256), 0, st, D, B, layer, kind,
+                     head, p0, n, out);
+  return launch_ex(k_kv_to_f32<float>, dim3(blocks), dim3(256), 0, st, D, B, layer, kind, head, p0,
+                   n, out);
 }
 
 }  // namespace ssd

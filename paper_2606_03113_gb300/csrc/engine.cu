@@ -10,6 +10,7 @@
 //   verify = embed(x, d_1..d_k) · layers(1..L) · head over k + 1 rows
 // Generation graph: WHILE(emitted < max_new) { round }.
 #include <stdio.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include <algorithm>
@@ -18,6 +19,7 @@
 #include <vector>
 
 #include "kernels.h"
+#include "pipe.cuh"
 
 using namespace ssd;
 
@@ -40,6 +42,7 @@ struct Carve {
 
 constexpr int kMaxQHidden = 1024;
 constexpr int kPrefillChunk = 16;
+constexpr int kMaxBlocks = 512;  // upper bound on the streamed kernels' grid (one block per SM)
 
 // Lays out every device buffer in the workspace; returns the total size.
 size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
@@ -56,22 +59,30 @@ size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
   d.kvd = c.n_kv_heads * c.head_dim;
   d.nsplit = (c.max_seq + kAttnChunk - 1) / kAttnChunk;
   d.eps = c.rms_eps;
-  d.res_blocks = (c.d_model / 2 + kWarps - 1) / kWarps;
+  d.num_sms = kMaxBlocks;  // set to the device's SM count at init
+  d.ss_tiles = (c.d_model + 15) / 16;
+  const int max_tiles = std::max(
+      std::max(head_tiles(c.vocab), c.ffn_dim / 8 + 1),
+      std::max((c.n_heads + 2 * c.n_kv_heads) * c.head_dim / 16 + 2, c.d_model / 16 + 1));
   const size_t elt = c.dtype == SSD_DTYPE_BF16 ? 2 : 4;
   Carve cv{base};
   Bufs b{};
   b.ctl = cv.take<Ctl>(sizeof(Ctl));
   b.h = cv.take<float>(sizeof(float) * kMaxM * d.d);
   b.ss = cv.take<float>(sizeof(float) * 2 * kMaxM);
-  b.ss_part = cv.take<float>(sizeof(float) * 2 * kMaxM * (size_t)d.res_blocks);
+  b.ss_tile = cv.take<float>(sizeof(float) * 2 * kMaxM * (size_t)d.ss_tiles);
   b.ss_counter = cv.take<uint32_t>(sizeof(uint32_t) * 2);
+  b.gpart = cv.take<float>(sizeof(float) * (size_t)kMaxBlocks * 2 * 16 * kMaxM);
+  b.tile_counter = cv.take<uint32_t>(sizeof(uint32_t) * (size_t)max_tiles);
+  b.head_group_counter = cv.take<uint32_t>(sizeof(uint32_t) * (size_t)head_groups(c.vocab));
   b.xq = cv.take<float>(sizeof(float) * kMaxM * d.qd);
   b.attn_part = cv.take<float>(sizeof(float) * kMaxM * d.Hq * (size_t)d.nsplit * d.hd);
   b.attn_ml = cv.take<float>(sizeof(float) * kMaxM * d.Hq * (size_t)d.nsplit * 2);
   b.attn_out = cv.take<float>(sizeof(float) * kMaxM * d.qd);
   b.act = cv.take<float>(sizeof(float) * kMaxM * d.F);
   b.logits = cv.take<float>(sizeof(float) * kMaxM * (size_t)d.V);
-  b.head_part = cv.take<void>(sizeof(HeadPart) * kMaxM * (size_t)head_blocks(d.V));
+  b.head_part = cv.take<void>(sizeof(HeadPart) * kMaxM *
+                              (size_t)(head_tiles(d.V) + head_groups(d.V)));
   b.head_counter = cv.take<uint32_t>(sizeof(uint32_t));
   b.stats = cv.take<RowStats>(sizeof(RowStats) * kMaxM);
   b.rope = cv.take<float2>(sizeof(float2) * (size_t)d.max_seq * (d.hd / 2));
@@ -167,6 +178,7 @@ struct Seq {
   cudaGraph_t g;
   cudaGraphNode_t last = nullptr;
   cudaError_t begin() {
+    g_pdl_ok = false;
     return cudaStreamBeginCaptureToGraph(x->cap, g, last ? &last : nullptr, nullptr, last ? 1 : 0,
                                          cudaStreamCaptureModeThreadLocal);
   }
@@ -403,9 +415,18 @@ ssd_status ssd_init_model(const ssd_model_cfg* cfg, const ssd_weights* w, void* 
   if (!workspace || ((uintptr_t)workspace & 255u))
     return fail(nullptr, SSD_ERR_INVALID_ARG, "workspace must be non-NULL and 256-byte aligned");
   if (workspace_bytes < need) return fail(nullptr, SSD_ERR_CAPACITY, "workspace too small");
+  if (cfg->head_dim % 32 || cfg->ffn_dim % 16)
+    return fail(nullptr, SSD_ERR_UNSUPPORTED, "head_dim must be a multiple of 32, ffn_dim of 16");
+  int dev = 0, sms = 0;
+  cudaError_t e0 = cudaGetDevice(&dev);
+  if (e0 == cudaSuccess) e0 = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e0 == cudaSuccess) e0 = prepare_gemv_kernels();
+  if (e0 != cudaSuccess) return cuda_fail(nullptr, "ssd_init_model device query", e0);
+  if (const char* v = getenv("SSD_NO_PDL")) g_pdl_enabled = !(v[0] == '1');
   ssd_ctx* x = new ssd_ctx();
   x->cfg = *cfg;
   layout(*cfg, static_cast<char*>(workspace), &x->D, &x->B);
+  x->D.num_sms = std::min(sms, kMaxBlocks);
   x->embed = w->embed;
   x->lm_head = w->lm_head;
   x->final_norm = w->final_norm;
@@ -435,6 +456,11 @@ ssd_status ssd_init_model(const ssd_model_cfg* cfg, const ssd_weights* w, void* 
   if (e == cudaSuccess) e = cudaMemsetAsync(x->B.head_counter, 0, sizeof(uint32_t), x->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(x->B.ss, 0, sizeof(float) * 2 * kMaxM, x->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(x->B.ss_counter, 0, sizeof(uint32_t) * 2, x->stream);
+  if (e == cudaSuccess)
+    e = cudaMemsetAsync(x->B.tile_counter, 0,
+                        (char*)x->B.head_group_counter - (char*)x->B.tile_counter +
+                            sizeof(uint32_t) * head_groups(cfg->vocab),
+                        x->stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(x->stream);
   if (e != cudaSuccess) {
     ssd_status s = cuda_fail(nullptr, "ssd_init_model upload", e);
@@ -771,7 +797,7 @@ ssd_status ssd_op_gemv(ssd_ctx* x, int32_t which, int32_t layer, int32_t M, cons
     default: return fail(x, SSD_ERR_INVALID_ARG, "which must be 0..4");
   }
   cudaStream_t st = stream ? static_cast<cudaStream_t>(stream) : x->stream;
-  CK(x, launch_gemv_plain(c.dtype, W, rows, cols, x_dev, M, y_dev, st));
+  CK(x, launch_gemv_plain(x->D, x->B, c.dtype, W, rows, cols, x_dev, M, y_dev, st));
   return SSD_OK;
 }
 

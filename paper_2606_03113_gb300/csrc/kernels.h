@@ -14,9 +14,10 @@ struct HeadPart {
   int32_t ti[kTopK];
 };
 
-constexpr int kHeadRowsPerBlock = 2 * kWarps;
-
-inline int head_blocks(int V) { return (V + kHeadRowsPerBlock - 1) / kHeadRowsPerBlock; }
+// Exit-head statistics partials: one per 16-row vocabulary tile and one per
+// group of 64 tiles.
+inline int head_tiles(int V) { return (V + 15) / 16; }
+inline int head_groups(int V) { return (head_tiles(V) + 63) / 64; }
 
 // big = true selects the kernels instantiated for up to kMaxM rows; false
 // the single-row ones.
@@ -45,8 +46,10 @@ cudaError_t launch_trace_push(const Bufs& B, int first_row, int n_rows, cudaStre
 cudaError_t launch_set_pending(const Bufs& B, int stats_row, int token, int pos, cudaStream_t st);
 cudaError_t launch_qnet_eval(const Bufs& B, int hidden, const float* states, int n, float* q,
                              cudaStream_t st);
-cudaError_t launch_gemv_plain(int dtype, const void* W, int rows, int cols, const float* x, int M,
-                              float* y, cudaStream_t st);
+cudaError_t launch_gemv_plain(const Dims& D, const Bufs& B, int dtype, const void* W, int rows,
+                              int cols, const float* x, int M, float* y, cudaStream_t st);
+// Raises the dynamic shared-memory limit of every streamed-kernel instance.
+cudaError_t prepare_gemv_kernels();
 cudaError_t launch_synth_fill(void* dst, int dtype, uint64_t n, uint32_t seed, uint32_t tid,
                               double sigma, cudaStream_t st);
 cudaError_t launch_read_probe(const void* src, uint64_t bytes, uint32_t* sink, cudaStream_t st);
