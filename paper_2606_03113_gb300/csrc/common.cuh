@@ -139,7 +139,7 @@ struct LayerW {
 
 // Shapes and buffers every kernel may need.
 struct Dims {
-  int32_t L, d, Hq, Hkv, hd, F, V, max_seq, qd, kvd, nsplit, num_sms, ss_tiles;
+  int32_t L, d, Hq, Hkv, hd, F, V, max_seq, qd, kvd, nsplit, num_sms, ss_tiles, max_tiles;
   float eps;
 };
 
@@ -147,19 +147,18 @@ struct Bufs {
   Ctl* ctl;
   float* h;          // [kMaxM][d] residual stream
   float* ss;         // [2][kMaxM] sum of squares of h rows: [0] after down/embed, [1] after O
-  float* ss_tile;    // [2][ss_tiles][kMaxM] per-tile partials of ss
-  uint32_t* ss_counter;  // [2] tile tickets of the residual kernels
+  float* ss_tile;    // [2][2][max blocks][kMaxM] per-block (running, split) partials of ss
+  uint32_t* ss_counter;  // [2] block tickets of the residual kernels
   float* gpart;      // [num_sms][2][32][kMaxM] partial tile sums of blocks sharing a tile
   uint32_t* tile_counter;      // [max tiles] tickets of shared tiles
-  uint32_t* head_group_counter;  // [head groups] tickets of the exit-head merge
   float* xq;         // [kMaxM][qd] rotated queries
   float* attn_part;  // [kMaxM][Hq][nsplit][hd] unnormalised partial outputs
   float* attn_ml;    // [kMaxM][Hq][nsplit][2] partial (max, sum)
   float* attn_out;   // [kMaxM][qd]
   float* act;        // [kMaxM][F]
   float* logits;     // [kMaxM][V] (written only when requested)
-  void* head_part;   // [head tiles + head groups][kMaxM] statistics partials
-  uint32_t* head_counter;
+  void* head_part;   // [2][max blocks][kMaxM] per-block (running, split) statistics
+  uint32_t* head_counter;  // block ticket of the exit head
   RowStats* stats;   // [kMaxM]
   float2* rope;      // [max_seq][hd/2] (cos, sin)
   void* kv;          // [L][2][Hkv][max_seq][hd]

@@ -42,7 +42,6 @@ struct Carve {
 
 constexpr int kMaxQHidden = 1024;
 constexpr int kPrefillChunk = 16;
-constexpr int kMaxBlocks = 512;  // upper bound on the streamed kernels' grid (one block per SM)
 
 // Lays out every device buffer in the workspace; returns the total size.
 size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
@@ -61,7 +60,7 @@ size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
   d.eps = c.rms_eps;
   d.num_sms = kMaxBlocks;  // set to the device's SM count at init
   d.ss_tiles = (c.d_model + 15) / 16;
-  const int max_tiles = std::max(
+  d.max_tiles = std::max(
       std::max(head_tiles(c.vocab), c.ffn_dim / 8 + 1),
       std::max((c.n_heads + 2 * c.n_kv_heads) * c.head_dim / 16 + 2, c.d_model / 16 + 1));
   const size_t elt = c.dtype == SSD_DTYPE_BF16 ? 2 : 4;
@@ -70,19 +69,18 @@ size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
   b.ctl = cv.take<Ctl>(sizeof(Ctl));
   b.h = cv.take<float>(sizeof(float) * kMaxM * d.d);
   b.ss = cv.take<float>(sizeof(float) * 2 * kMaxM);
-  b.ss_tile = cv.take<float>(sizeof(float) * 2 * kMaxM * (size_t)d.ss_tiles);
+  b.ss_tile = cv.take<float>(sizeof(float) * 2 * 2 * kMaxM * (size_t)kMaxBlocks);
   b.ss_counter = cv.take<uint32_t>(sizeof(uint32_t) * 2);
   b.gpart = cv.take<float>(sizeof(float) * (size_t)kMaxBlocks * 2 * 16 * kMaxM);
-  b.tile_counter = cv.take<uint32_t>(sizeof(uint32_t) * (size_t)max_tiles);
-  b.head_group_counter = cv.take<uint32_t>(sizeof(uint32_t) * (size_t)head_groups(c.vocab));
+  b.tile_counter = cv.take<uint32_t>(sizeof(uint32_t) * (size_t)d.max_tiles);
+
   b.xq = cv.take<float>(sizeof(float) * kMaxM * d.qd);
   b.attn_part = cv.take<float>(sizeof(float) * kMaxM * d.Hq * (size_t)d.nsplit * d.hd);
   b.attn_ml = cv.take<float>(sizeof(float) * kMaxM * d.Hq * (size_t)d.nsplit * 2);
   b.attn_out = cv.take<float>(sizeof(float) * kMaxM * d.qd);
   b.act = cv.take<float>(sizeof(float) * kMaxM * d.F);
   b.logits = cv.take<float>(sizeof(float) * kMaxM * (size_t)d.V);
-  b.head_part = cv.take<void>(sizeof(HeadPart) * kMaxM *
-                              (size_t)(head_tiles(d.V) + head_groups(d.V)));
+  b.head_part = cv.take<void>(sizeof(HeadPart) * kMaxM * 2 * (size_t)kMaxBlocks);
   b.head_counter = cv.take<uint32_t>(sizeof(uint32_t));
   b.stats = cv.take<RowStats>(sizeof(RowStats) * kMaxM);
   b.rope = cv.take<float2>(sizeof(float2) * (size_t)d.max_seq * (d.hd / 2));
@@ -457,10 +455,7 @@ ssd_status ssd_init_model(const ssd_model_cfg* cfg, const ssd_weights* w, void* 
   if (e == cudaSuccess) e = cudaMemsetAsync(x->B.ss, 0, sizeof(float) * 2 * kMaxM, x->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(x->B.ss_counter, 0, sizeof(uint32_t) * 2, x->stream);
   if (e == cudaSuccess)
-    e = cudaMemsetAsync(x->B.tile_counter, 0,
-                        (char*)x->B.head_group_counter - (char*)x->B.tile_counter +
-                            sizeof(uint32_t) * head_groups(cfg->vocab),
-                        x->stream);
+    e = cudaMemsetAsync(x->B.tile_counter, 0, sizeof(uint32_t) * (size_t)x->D.max_tiles, x->stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(x->stream);
   if (e != cudaSuccess) {
     ssd_status s = cuda_fail(nullptr, "ssd_init_model upload", e);

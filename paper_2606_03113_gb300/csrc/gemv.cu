@@ -41,7 +41,7 @@ constexpr int kCWarps = 8;          // consumer warps
 constexpr int kCThreads = kCWarps * 32;
 constexpr int kThreads = kCThreads + 32;  // + producer warp
 constexpr int kStageBytes = kRT * kRowBytes;
-constexpr int kGroupTiles = 64;     // exit-head tiles merged per group
+constexpr int kMaxBlocksDev = 512;  // upper bound on the grid (partial slots per block)
 
 enum RowMap : int { kMapLinear = 0, kMapQKV = 1, kMapGateUp = 2 };
 
@@ -110,26 +110,36 @@ __device__ __forceinline__ int warp_row(int w, int i) { return w + 8 * i; }
 struct SmemLayout {
   static constexpr size_t ring = 0;
   static constexpr size_t bars = ring + (size_t)kNS * kStageBytes;
-  static constexpr size_t tile = bars + 2 * kNS * sizeof(uint64_t);
+  static constexpr size_t rs = bars + 2 * kNS * sizeof(uint64_t);
+  static constexpr size_t flag = rs + sizeof(float) * 32;
+  static constexpr size_t scratch = flag + 64;  // cross-warp combine buffer
+  // combine buffers are indexed [warp][kMaxM] whatever MM is
   template <int MM>
-  static constexpr size_t aux() { return tile + sizeof(float) * kRT * MM; }
-  template <int MM>
-  static constexpr size_t rs() { return aux<MM>() + sizeof(float) * kRT * MM; }
-  template <int MM>
-  static constexpr size_t flag() { return rs<MM>() + sizeof(float) * 32; }
-  template <int MM>
-  static constexpr size_t total() { return flag<MM>() + 64; }
+  static constexpr size_t total() { return scratch + (size_t)kCWarps * kMaxM * sizeof(HeadPart); }
 };
 
-struct TileCtx {
-  float* sum;   // [16][MM] tile sums
-  float* aux;   // [16][MM] scratch
-  float* rs;    // [MM] input RMSNorm scale
+// Block b owns the exit-head / norm partial of the tile it starts and shares
+// with the next block(s) ("split slot"), if its last tile is such a tile.
+__device__ inline bool has_split_slot(const Geom& g, int b) {
+  const long long sb = stage_start(g, b), se = stage_start(g, b + 1);
+  if (se <= sb) return false;
+  const long long t = (se - 1) / g.nks;
+  if ((t + 1) * g.nks <= se) return false;  // the last tile ends inside the block
+  return t * g.nks >= sb;                   // and it starts inside the block
+}
+
+struct Shared {
+  float* rs;       // [MM] input RMSNorm scale
   int* flag;
-  int M, pos0, tid;
+  void* scratch;   // [kCWarps][MM] floats or HeadParts
 };
 
 // ------------------------------------------------------------ epilogues
+//
+// pair(): rows (w, w+8) of a tile, one input row m per lane (lane < M), with
+// the dot products v0, v1.  Kernels with a running result (residual norm sums,
+// exit-head statistics) keep per-lane state; finish() combines it once per
+// block and the last block reduces the blocks in a fixed order.
 
 __device__ __forceinline__ bool better(float v1, int i1, float v2, int i2) {
   return v1 > v2 || (v1 == v2 && i1 < i2);
@@ -144,18 +154,6 @@ __device__ inline void part_empty(HeadPart& p) {
     p.tv[q] = -INFINITY;
     p.ti[q] = 0x7fffffff;
   }
-}
-
-__device__ inline void part_insert_topk(HeadPart& p, float v, int idx) {
-  if (!better(v, idx, p.tv[kTopK - 1], p.ti[kTopK - 1])) return;
-  int q = kTopK - 1;
-  while (q > 0 && better(v, idx, p.tv[q - 1], p.ti[q - 1])) {
-    p.tv[q] = p.tv[q - 1];
-    p.ti[q] = p.ti[q - 1];
-    --q;
-  }
-  p.tv[q] = v;
-  p.ti[q] = idx;
 }
 
 // a <- merge(a, b); symmetric in a and b (max, commutative sums, ordered
@@ -194,6 +192,36 @@ __device__ inline void part_merge(HeadPart& a, const HeadPart& b) {
   }
 }
 
+// Adds one logit z of vocabulary row idx.
+__device__ inline void part_add(HeadPart& p, float z, int idx) {
+  if (!(z > -INFINITY)) return;
+  if (p.S > 0.f) {
+    if (z > p.mx) {
+      const float e = expf(p.mx - z);
+      p.T = e * (p.T + (p.mx - z) * p.S);
+      p.S = p.S * e + 1.f;
+      p.mx = z;
+    } else {
+      const float e = expf(z - p.mx);
+      p.S += e;
+      p.T += e * (z - p.mx);
+    }
+  } else {
+    p.mx = z;
+    p.S = 1.f;
+    p.T = 0.f;
+  }
+  if (!better(z, idx, p.tv[kTopK - 1], p.ti[kTopK - 1])) return;
+  int q = kTopK - 1;
+  while (q > 0 && better(z, idx, p.tv[q - 1], p.ti[q - 1])) {
+    p.tv[q] = p.tv[q - 1];
+    p.ti[q] = p.ti[q - 1];
+    --q;
+  }
+  p.tv[q] = z;
+  p.ti[q] = idx;
+}
+
 __device__ inline HeadPart part_shfl(const HeadPart& p, int off) {
   HeadPart q;
   q.mx = __shfl_xor_sync(0xffffffffu, p.mx, off);
@@ -220,202 +248,226 @@ __device__ inline HeadPart part_load_cg(const HeadPart* src) {
   return q;
 }
 
+struct NoState {};
+
 // y[m][row] = sum (the plain product, for kernel-level parity and timing).
 struct EpiPlain {
+  using State = NoState;
   float* y;
-  template <int MM>
-  __device__ void apply(const StreamArgs& a, int tile, const TileCtx& c) const {
-    for (int idx = c.tid; idx < kRT * c.M; idx += kCThreads) {
-      const int r = idx / c.M, m = idx - r * c.M;
-      const int row = map_row(a.g, a.D, tile, r);
-      if (row >= 0) y[(size_t)m * a.g.N + row] = c.sum[r * MM + m];
-    }
+  __device__ void init(State&) const {}
+  __device__ void pair(const StreamArgs& a, int tile, int w, int m, int, float, float v0, float v1,
+                       State&) const {
+    const int r0 = map_row(a.g, a.D, tile, w), r1 = map_row(a.g, a.D, tile, w + 8);
+    if (r0 >= 0) y[(size_t)m * a.g.N + r0] = v0;
+    if (r1 >= 0) y[(size_t)m * a.g.N + r1] = v1;
   }
+  __device__ void split_done(const StreamArgs&, int, State&, const Shared&, int, int) const {}
+  __device__ void finish(const StreamArgs&, State&, const Shared&, int, int) const {}
 };
 
 // Rotary embedding of query/key pairs (element i with i + hd/2, angle
-// pos * theta^(-2i/hd) from the table), queries to xq, keys and values to
+// pos * theta^(-2i/hd) from the table); queries to xq, keys and values to
 // the KV cache of `layer` at positions pos0 + m.
 template <typename T>
 struct EpiQKV {
+  using State = NoState;
   int layer;
-  template <int MM>
-  __device__ void apply(const StreamArgs& a, int tile, const TileCtx& c) const {
+  __device__ void init(State&) const {}
+  __device__ void pair(const StreamArgs& a, int tile, int w, int m, int pos0, float rs, float v0,
+                       float v1, State&) const {
     const Dims& D = a.D;
     const int tqk = (D.Hq + D.Hkv) * (D.hd / 16);
     T* kv = static_cast<T*>(a.B.kv) + (size_t)layer * 2 * D.Hkv * D.max_seq * D.hd;
-    const int half = D.hd / 2;
-    for (int idx = c.tid; idx < 8 * c.M; idx += kCThreads) {
-      const int p = idx / c.M, m = idx - p * c.M;
-      const int pos = c.pos0 + m;
-      const float y0 = c.sum[p * MM + m] * c.rs[m];
-      const float y1 = c.sum[(p + 8) * MM + m] * c.rs[m];
-      const int r0 = map_row(a.g, D, tile, p);
-      if (tile < tqk) {
-        const int head = r0 / D.hd, i = r0 - head * D.hd;
-        const float2 cs = a.B.rope[(size_t)pos * half + i];
-        const float o0 = y0 * cs.x - y1 * cs.y;
-        const float o1 = y1 * cs.x + y0 * cs.y;
-        if (head < D.Hq) {
-          float* q = a.B.xq + (size_t)m * D.qd + (size_t)head * D.hd;
-          q[i] = o0;
-          q[i + half] = o1;
-        } else {
-          T* kr = kv + ((size_t)(head - D.Hq) * D.max_seq + pos) * D.hd;
-          kr[i] = Elem<T>::from_f(o0);
-          kr[i + half] = Elem<T>::from_f(o1);
-        }
+    const int pos = pos0 + m;
+    const float y0 = v0 * rs, y1 = v1 * rs;
+    const int r0 = map_row(a.g, D, tile, w);
+    if (tile < tqk) {
+      const int half = D.hd / 2;
+      const int head = r0 / D.hd, i = r0 - head * D.hd;
+      const float2 cs = a.B.rope[(size_t)pos * half + i];
+      const float o0 = y0 * cs.x - y1 * cs.y;
+      const float o1 = y1 * cs.x + y0 * cs.y;
+      if (head < D.Hq) {
+        float* q = a.B.xq + (size_t)m * D.qd + (size_t)head * D.hd;
+        q[i] = o0;
+        q[i + half] = o1;
       } else {
-        const int r1 = map_row(a.g, D, tile, p + 8);
-        const int vb = (D.Hq + D.Hkv) * D.hd;
-        if (r0 >= 0) {
-          const int g = (r0 - vb) / D.hd, j = (r0 - vb) - g * D.hd;
-          kv[((size_t)(D.Hkv + g) * D.max_seq + pos) * D.hd + j] = Elem<T>::from_f(y0);
-        }
-        if (r1 >= 0) {
-          const int g = (r1 - vb) / D.hd, j = (r1 - vb) - g * D.hd;
-          kv[((size_t)(D.Hkv + g) * D.max_seq + pos) * D.hd + j] = Elem<T>::from_f(y1);
-        }
+        T* kr = kv + ((size_t)(head - D.Hq) * D.max_seq + pos) * D.hd;
+        kr[i] = Elem<T>::from_f(o0);
+        kr[i + half] = Elem<T>::from_f(o1);
+      }
+    } else {
+      const int r1 = map_row(a.g, D, tile, w + 8);
+      const int vb = (D.Hq + D.Hkv) * D.hd;
+      if (r0 >= 0) {
+        const int g = (r0 - vb) / D.hd, j = (r0 - vb) - g * D.hd;
+        kv[((size_t)(D.Hkv + g) * D.max_seq + pos) * D.hd + j] = Elem<T>::from_f(y0);
+      }
+      if (r1 >= 0) {
+        const int g = (r1 - vb) / D.hd, j = (r1 - vb) - g * D.hd;
+        kv[((size_t)(D.Hkv + g) * D.max_seq + pos) * D.hd + j] = Elem<T>::from_f(y1);
       }
     }
   }
+  __device__ void split_done(const StreamArgs&, int, State&, const Shared&, int, int) const {}
+  __device__ void finish(const StreamArgs&, State&, const Shared&, int, int) const {}
 };
 
 // act[m][j] = silu(gate_j) * up_j.
 struct EpiGateUp {
-  template <int MM>
-  __device__ void apply(const StreamArgs& a, int tile, const TileCtx& c) const {
-    const int F = a.D.F;
-    for (int idx = c.tid; idx < 8 * c.M; idx += kCThreads) {
-      const int p = idx / c.M, m = idx - p * c.M;
-      const int j = map_row(a.g, a.D, tile, p);
-      if (j < 0) continue;
-      const float gt = c.sum[p * MM + m] * c.rs[m];
-      const float up = c.sum[(p + 8) * MM + m] * c.rs[m];
-      a.B.act[(size_t)m * F + j] = gt / (1.0f + expf(-gt)) * up;
-    }
+  using State = NoState;
+  __device__ void init(State&) const {}
+  __device__ void pair(const StreamArgs& a, int tile, int w, int m, int, float rs, float v0,
+                       float v1, State&) const {
+    const int j = map_row(a.g, a.D, tile, w);
+    if (j < 0) return;
+    const float gt = v0 * rs, up = v1 * rs;
+    a.B.act[(size_t)m * a.D.F + j] = gt / (1.0f + expf(-gt)) * up;
   }
+  __device__ void split_done(const StreamArgs&, int, State&, const Shared&, int, int) const {}
+  __device__ void finish(const StreamArgs&, State&, const Shared&, int, int) const {}
 };
 
-// h[m][row] += y; sum(h_m^2) for the next RMSNorm: each tile's sum goes to a
-// per-tile slot, and the last tile to finish adds the slots in tile order.
+// Combines the per-lane float state of the 8 warps (lane m of each) in warp
+// order; every consumer thread calls it; returns the sum in thread m < M.
+__device__ inline float combine_warps(float v, const Shared& sh, int tid, int M) {
+  float* buf = static_cast<float*>(sh.scratch);
+  const int warp = tid >> 5, lane = tid & 31;
+  if (lane < M) buf[warp * kMaxM + lane] = v;
+  named_sync(1, kCThreads);
+  float s = 0.f;
+  if (tid < M)
+    for (int w = 0; w < kCWarps; ++w) s += buf[w * kMaxM + tid];
+  named_sync(1, kCThreads);
+  return s;
+}
+
+// h[m][row] += y, and sum(h_m^2) over the rows for the next RMSNorm.  Per
+// block: one running sum (complete tiles) and one split-slot sum (the tile it
+// starts and shares); the last block adds them in block order.
 struct EpiResid {
+  struct State {
+    float ss;
+  };
   int which;  // sum-of-squares buffer written (0 after down, 1 after O)
-  template <int MM>
-  __device__ void apply(const StreamArgs& a, int tile, const TileCtx& c) const {
-    const Dims& D = a.D;
-    for (int idx = c.tid; idx < kRT * c.M; idx += kCThreads) {
-      const int r = idx / c.M, m = idx - r * c.M;
-      const int row = map_row(a.g, D, tile, r);
-      float sq = 0.f;
-      if (row >= 0) {
-        float* hp = a.B.h + (size_t)m * D.d + row;
-        const float v = *hp + c.sum[r * MM + m];
-        *hp = v;
-        sq = v * v;
+  __device__ void init(State& s) const { s.ss = 0.f; }
+  __device__ void pair(const StreamArgs& a, int tile, int w, int m, int, float, float v0, float v1,
+                       State& st) const {
+    const int r0 = map_row(a.g, a.D, tile, w), r1 = map_row(a.g, a.D, tile, w + 8);
+    float* hm = a.B.h + (size_t)m * a.D.d;
+    if (r0 >= 0) {
+      const float h = hm[r0] + v0;
+      hm[r0] = h;
+      st.ss = fmaf(h, h, st.ss);
+    }
+    if (r1 >= 0) {
+      const float h = hm[r1] + v1;
+      hm[r1] = h;
+      st.ss = fmaf(h, h, st.ss);
+    }
+  }
+  __device__ float* slots(const StreamArgs& a) const {
+    return a.B.ss_tile + (size_t)which * 2 * kMaxBlocksDev * kMaxM;
+  }
+  __device__ void split_done(const StreamArgs& a, int b0, State& st, const Shared& sh, int tid,
+                             int M) const {
+    const float s = combine_warps(st.ss, sh, tid, M);
+    if (tid < M) slots(a)[((size_t)kMaxBlocksDev + b0) * kMaxM + tid] = s;
+  }
+  __device__ void finish(const StreamArgs& a, State& st, const Shared& sh, int tid, int M) const {
+    const float s = combine_warps(st.ss, sh, tid, M);
+    float* sl = slots(a);
+    if (tid < M) sl[(size_t)blockIdx.x * kMaxM + tid] = s;
+    __threadfence();
+    named_sync(1, kCThreads);
+    if (tid == 0) *sh.flag = atomicAdd(&a.B.ss_counter[which], 1u) == (unsigned)(a.g.P - 1);
+    named_sync(1, kCThreads);
+    if (!*sh.flag) return;
+    __threadfence();
+    const int warp = tid >> 5, lane = tid & 31;
+    for (int m = warp; m < M; m += kCWarps) {
+      float v = 0.f;
+      for (int b = lane; b < a.g.P; b += 32) {
+        v += __ldcg(&sl[(size_t)b * kMaxM + m]);
+        if (has_split_slot(a.g, b)) v += __ldcg(&sl[((size_t)kMaxBlocksDev + b) * kMaxM + m]);
       }
-      c.aux[r * MM + m] = sq;
+      v = warp_sum(v);
+      if (lane == 0) a.B.ss[which * kMaxM + m] = v;
     }
-    named_sync(1, kCThreads);
-    float* slots = a.B.ss_tile + (size_t)which * D.ss_tiles * kMaxM;
-    if (c.tid < c.M) {
-      float s = 0.f;
-      for (int r = 0; r < kRT; ++r) s += c.aux[r * MM + c.tid];
-      slots[(size_t)tile * kMaxM + c.tid] = s;
-    }
-    __threadfence();
-    named_sync(1, kCThreads);
-    if (c.tid == 0)
-      *c.flag = atomicAdd(&a.B.ss_counter[which], 1u) == (unsigned)(a.g.ntiles - 1);
-    named_sync(1, kCThreads);
-    if (!*c.flag) return;
-    __threadfence();
-    const int warp = c.tid >> 5, lane = c.tid & 31;
-    for (int m = warp; m < c.M; m += kCWarps) {
-      float s = 0.f;
-      for (int t = lane; t < a.g.ntiles; t += 32) s += __ldcg(&slots[(size_t)t * kMaxM + m]);
-      s = warp_sum(s);
-      if (lane == 0) a.B.ss[which * kMaxM + m] = s;
-    }
-    if (c.tid == 0) a.B.ss_counter[which] = 0u;
+    if (tid == 0) a.B.ss_counter[which] = 0u;
   }
 };
 
-// Exit head: z = W_lm RMSNorm_final(h).  Per tile, a statistics partial
-// (max, sum exp, sum exp*(z-max), top-k); groups of 64 tiles are merged by the
-// group's last finisher, and the groups by the last group (a fixed shuffle
-// tree), giving argmax (lowest id on ties), log-sum-exp, entropy
-// H = log S - T/S, C_k = lse - mean(top-k logits), pmax = 1/S.
+// Merges the per-lane statistics of the 8 warps (lane m of each) in warp
+// order; result in thread m < M.
+__device__ inline HeadPart combine_parts(const HeadPart& p, const Shared& sh, int tid, int M) {
+  HeadPart* buf = static_cast<HeadPart*>(sh.scratch);
+  const int warp = tid >> 5, lane = tid & 31;
+  if (lane < M) buf[warp * kMaxM + lane] = p;
+  named_sync(1, kCThreads);
+  HeadPart r;
+  part_empty(r);
+  if (tid < M)
+    for (int w = 0; w < kCWarps; ++w) part_merge(r, buf[w * kMaxM + tid]);
+  named_sync(1, kCThreads);
+  return r;
+}
+
+// Exit head: z = W_lm RMSNorm_final(h).  Lane m keeps running statistics of
+// the logits it produced (max, sum exp, sum exp*(z-max), top-k); per block
+// they are merged in warp order, and the last block merges the blocks (and
+// the split slots) in a fixed shuffle tree, giving argmax (lowest id on
+// ties), log-sum-exp, entropy H = log S - T/S, C_k = lse - mean(top-k
+// logits) and pmax = 1/S.
 struct EpiHead {
+  struct State {
+    HeadPart p;
+  };
   int topk, write_logits;
-  template <int MM>
-  __device__ void apply(const StreamArgs& a, int tile, const TileCtx& c) const {
-    const Dims& D = a.D;
-    const Bufs& B = a.B;
-    for (int idx = c.tid; idx < kRT * c.M; idx += kCThreads) {
-      const int r = idx / c.M, m = idx - r * c.M;
-      const int row = map_row(a.g, D, tile, r);
-      const float z = row >= 0 ? c.sum[r * MM + m] * c.rs[m] : -INFINITY;
-      c.aux[r * MM + m] = z;
-      if (write_logits && row >= 0) B.logits[(size_t)m * D.V + row] = z;
+  __device__ void init(State& s) const { part_empty(s.p); }
+  __device__ void pair(const StreamArgs& a, int tile, int w, int m, int, float rs, float v0,
+                       float v1, State& st) const {
+    const int r0 = map_row(a.g, a.D, tile, w), r1 = map_row(a.g, a.D, tile, w + 8);
+    if (r0 >= 0) {
+      const float z = v0 * rs;
+      part_add(st.p, z, r0);
+      if (write_logits) a.B.logits[(size_t)m * a.D.V + r0] = z;
     }
+    if (r1 >= 0) {
+      const float z = v1 * rs;
+      part_add(st.p, z, r1);
+      if (write_logits) a.B.logits[(size_t)m * a.D.V + r1] = z;
+    }
+  }
+  __device__ HeadPart* slots(const StreamArgs& a) const {
+    return static_cast<HeadPart*>(a.B.head_part);
+  }
+  __device__ void split_done(const StreamArgs& a, int b0, State& st, const Shared& sh, int tid,
+                             int M) const {
+    const HeadPart r = combine_parts(st.p, sh, tid, M);
+    if (tid < M) slots(a)[((size_t)kMaxBlocksDev + b0) * kMaxM + tid] = r;
+  }
+  __device__ void finish(const StreamArgs& a, State& st, const Shared& sh, int tid, int M) const {
+    const HeadPart r = combine_parts(st.p, sh, tid, M);
+    HeadPart* sl = slots(a);
+    if (tid < M) sl[(size_t)blockIdx.x * kMaxM + tid] = r;
+    __threadfence();
     named_sync(1, kCThreads);
-    HeadPart* tiles = static_cast<HeadPart*>(B.head_part);
-    HeadPart* groups = tiles + (size_t)a.g.ntiles * kMaxM;
-    if (c.tid < c.M) {
+    if (tid == 0) *sh.flag = atomicAdd(a.B.head_counter, 1u) == (unsigned)(a.g.P - 1);
+    named_sync(1, kCThreads);
+    if (!*sh.flag) return;
+    __threadfence();
+    const int warp = tid >> 5, lane = tid & 31;
+    for (int m = warp; m < M; m += kCWarps) {
       HeadPart p;
       part_empty(p);
-      float mx = -INFINITY;
-      for (int r = 0; r < kRT; ++r) mx = fmaxf(mx, c.aux[r * MM + c.tid]);
-      if (mx > -INFINITY) {
-        float S = 0.f, Tt = 0.f;
-        for (int r = 0; r < kRT; ++r) {
-          const float z = c.aux[r * MM + c.tid];
-          if (z > -INFINITY) {
-            const float e = expf(z - mx);
-            S += e;
-            Tt += e * (z - mx);
-            part_insert_topk(p, z, tile * kRT + r);
-          }
-        }
-        p.mx = mx;
-        p.S = S;
-        p.T = Tt;
+      for (int b = lane; b < a.g.P; b += 32) {
+        part_merge(p, part_load_cg(&sl[(size_t)b * kMaxM + m]));
+        if (has_split_slot(a.g, b)) part_merge(p, part_load_cg(&sl[((size_t)kMaxBlocksDev + b) * kMaxM + m]));
       }
-      tiles[(size_t)tile * kMaxM + c.tid] = p;
-    }
-    __threadfence();
-    named_sync(1, kCThreads);
-    const int grp = tile / kGroupTiles;
-    const int g0 = grp * kGroupTiles, g1 = min(a.g.ntiles, g0 + kGroupTiles);
-    if (c.tid == 0)
-      *c.flag = atomicAdd(&B.head_group_counter[grp], 1u) == (unsigned)(g1 - g0 - 1);
-    named_sync(1, kCThreads);
-    if (!*c.flag) return;
-    __threadfence();
-    const int warp = c.tid >> 5, lane = c.tid & 31;
-    for (int m = warp; m < c.M; m += kCWarps) {  // group merge: lanes, then a shuffle tree
-      HeadPart p;
-      part_empty(p);
-      for (int t = g0 + lane; t < g1; t += 32) part_merge(p, part_load_cg(&tiles[(size_t)t * kMaxM + m]));
-      for (int off = 16; off > 0; off >>= 1) part_merge(p, part_shfl(p, off));
-      if (lane == 0) groups[(size_t)grp * kMaxM + m] = p;
-    }
-    if (c.tid == 0) B.head_group_counter[grp] = 0u;
-    __threadfence();
-    named_sync(1, kCThreads);
-    const int ngroups = (a.g.ntiles + kGroupTiles - 1) / kGroupTiles;
-    if (c.tid == 0) *c.flag = atomicAdd(B.head_counter, 1u) == (unsigned)(ngroups - 1);
-    named_sync(1, kCThreads);
-    if (!*c.flag) return;
-    __threadfence();
-    for (int m = warp; m < c.M; m += kCWarps) {
-      HeadPart p;
-      part_empty(p);
-      for (int t = lane; t < ngroups; t += 32) part_merge(p, part_load_cg(&groups[(size_t)t * kMaxM + m]));
       for (int off = 16; off > 0; off >>= 1) part_merge(p, part_shfl(p, off));
       if (lane == 0) {
-        RowStats& o = B.stats[m];
+        RowStats& o = a.B.stats[m];
         const float logS = logf(p.S);
         o.argmax = p.ti[0];
         o.zmax = p.mx;
@@ -432,11 +484,20 @@ struct EpiHead {
         o.margin = p.tv[0] - p.tv[1];
       }
     }
-    if (c.tid == 0) *B.head_counter = 0u;
+    if (tid == 0) *a.B.head_counter = 0u;
   }
 };
 
 // ------------------------------------------------------------ the kernel
+
+template <int MM>
+__device__ __forceinline__ float pick(const float (&v)[MM], int lane) {
+  float r = 0.f;
+#pragma unroll
+  for (int m = 0; m < MM; ++m)
+    if (m == lane) r = v[m];
+  return r;
+}
 
 template <typename T, int MM, class Epi>
 __global__ void __launch_bounds__(kThreads, 1) k_stream(const StreamArgs a, const Epi epi) {
@@ -446,10 +507,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_stream(const StreamArgs a, cons
   unsigned char* ring = smem + SmemLayout::ring;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + SmemLayout::bars);
   uint64_t* empty = full + kNS;
-  float* sm_sum = reinterpret_cast<float*>(smem + SmemLayout::tile);
-  float* sm_aux = reinterpret_cast<float*>(smem + SmemLayout::aux<MM>());
-  float* sm_rs = reinterpret_cast<float*>(smem + SmemLayout::rs<MM>());
-  int* sm_flag = reinterpret_cast<int*>(smem + SmemLayout::flag<MM>());
+  const Shared sh{reinterpret_cast<float*>(smem + SmemLayout::rs),
+                  reinterpret_cast<int*>(smem + SmemLayout::flag), smem + SmemLayout::scratch};
 
   const Geom& g = a.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -499,20 +558,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_stream(const StreamArgs a, cons
   int pos0, M;
   resolve_rows(a.B.ctl, a.sel, pos0, M);
   const int tid = threadIdx.x;
-  if (tid < MM) {
+  if (tid < 32) {
     float r = 1.f;
     if (a.ss_in >= 0 && tid < M) r = 1.0f / sqrtf(a.B.ss[a.ss_in * kMaxM + tid] / (float)g.K + a.D.eps);
-    sm_rs[tid] = r;
+    sh.rs[tid] = r;
   }
   named_sync(1, kCThreads);
-  const TileCtx tc{sm_sum, sm_aux, sm_rs, sm_flag, M, pos0, tid};
+  const float my_rs = sh.rs[lane];
   const float* x = a.x;
   const T* gn = static_cast<const T*>(a.gnorm);
   const int KC = kRowBytes / (int)sizeof(T);
+  typename Epi::State run;
+  epi.init(run);
   float acc[2][MM];
-  int rloc[2];
-#pragma unroll
-  for (int i = 0; i < 2; ++i) rloc[i] = warp_row(warp, i);
+  const int rloc[2] = {warp, warp + 8};
   int cur = -1;
   bool ok = true;
   for (long long s = s_begin; s < s_end; ++s) {
@@ -572,54 +631,53 @@ __global__ void __launch_bounds__(kThreads, 1) k_stream(const StreamArgs a, cons
     if (lane == 0) mbar_arrive(&empty[slot]);
     if (ks != g.nks - 1 && s != s_end - 1) continue;
 
-    // ---- tile flush (all consumer warps together)
+    // ---- tile flush: warp-local unless the tile is shared with other blocks
+    float v[2][MM];
 #pragma unroll
     for (int r = 0; r < 2; ++r)
 #pragma unroll
-      for (int m = 0; m < MM; ++m)
-        if (m < M) {
-          const float v = warp_sum(acc[r][m]);
-          if (lane == 0) sm_sum[rloc[r] * MM + m] = v;
-        }
-    named_sync(1, kCThreads);
+      for (int m = 0; m < MM; ++m) v[r][m] = m < M ? warp_sum(acc[r][m]) : 0.f;
     const long long t0 = (long long)tile * g.nks, t1 = t0 + g.nks;
-    if (t0 < s_begin || t1 > s_end) {
-      // shared with neighbouring blocks: publish this block's partial
-      const int first_tile = (int)(s_begin / g.nks);
-      const int slot2 = tile == first_tile ? 0 : 1;
-      float* mine = a.B.gpart + ((size_t)blockIdx.x * 2 + slot2) * kRT * kMaxM;
-      for (int idx = tid; idx < kRT * M; idx += kCThreads) {
-        const int r = idx / M, m = idx - r * M;
-        mine[r * kMaxM + m] = sm_sum[r * MM + m];
-      }
-      __threadfence();
-      named_sync(1, kCThreads);
-      const int b0 = block_of_stage(g, t0), b1 = block_of_stage(g, t1 - 1);
-      if (tid == 0) {
-        int contrib = 0;
-        for (int b = b0; b <= b1; ++b) contrib += stage_start(g, b) < stage_start(g, b + 1);
-        *sm_flag = atomicAdd(&a.B.tile_counter[tile], 1u) == (unsigned)(contrib - 1);
-      }
-      named_sync(1, kCThreads);
-      if (!*sm_flag) continue;
-      __threadfence();
-      for (int idx = tid; idx < kRT * M; idx += kCThreads) {
-        const int r = idx / M, m = idx - r * M;
-        float v = 0.f;
-        for (int b = b0; b <= b1; ++b) {
-          const long long sb = stage_start(g, b);
-          if (sb == stage_start(g, b + 1)) continue;
-          const int sl = tile == (int)(sb / g.nks) ? 0 : 1;
-          v += __ldcg(&a.B.gpart[((size_t)b * 2 + sl) * kRT * kMaxM + r * kMaxM + m]);
-        }
-        sm_sum[r * MM + m] = v;
-      }
-      if (tid == 0) a.B.tile_counter[tile] = 0u;
-      named_sync(1, kCThreads);
+    if (t0 >= s_begin && t1 <= s_end) {
+      if (lane < M) epi.pair(a, tile, warp, lane, pos0, my_rs, pick(v[0], lane), pick(v[1], lane), run);
+      continue;
     }
-    epi.template apply<MM>(a, tile, tc);
+    // shared with neighbouring blocks: publish this block's partial sums
+    const int first_tile = (int)(s_begin / g.nks);
+    const int slot2 = tile == first_tile ? 0 : 1;
+    float* mine = a.B.gpart + ((size_t)blockIdx.x * 2 + slot2) * kRT * kMaxM;
+    if (lane < M) {
+      mine[rloc[0] * kMaxM + lane] = pick(v[0], lane);
+      mine[rloc[1] * kMaxM + lane] = pick(v[1], lane);
+    }
+    __threadfence();
     named_sync(1, kCThreads);
+    const int b0 = block_of_stage(g, t0), b1 = block_of_stage(g, t1 - 1);
+    if (tid == 0) {
+      int contrib = 0;
+      for (int b = b0; b <= b1; ++b) contrib += stage_start(g, b) < stage_start(g, b + 1);
+      *sh.flag = atomicAdd(&a.B.tile_counter[tile], 1u) == (unsigned)(contrib - 1);
+    }
+    named_sync(1, kCThreads);
+    if (!*sh.flag) continue;
+    __threadfence();
+    float u0 = 0.f, u1 = 0.f;
+    if (lane < M)
+      for (int b = b0; b <= b1; ++b) {  // block order: independent of who finishes
+        const long long sb = stage_start(g, b);
+        if (sb == stage_start(g, b + 1)) continue;
+        const int sl = tile == (int)(sb / g.nks) ? 0 : 1;
+        const float* p = a.B.gpart + ((size_t)b * 2 + sl) * kRT * kMaxM;
+        u0 += __ldcg(&p[rloc[0] * kMaxM + lane]);
+        u1 += __ldcg(&p[rloc[1] * kMaxM + lane]);
+      }
+    if (tid == 0) a.B.tile_counter[tile] = 0u;
+    typename Epi::State sp;
+    epi.init(sp);
+    if (lane < M) epi.pair(a, tile, warp, lane, pos0, my_rs, u0, u1, sp);
+    epi.split_done(a, b0, sp, sh, tid, M);
   }
+  epi.finish(a, run, sh, tid, M);
 }
 
 // ------------------------------------------------------------- launchers
@@ -655,6 +713,7 @@ static cudaError_t stream_launch(const StreamArgs& a, const Epi& epi, cudaStream
 
 template <typename T, int MM, class Epi>
 static cudaError_t prepare_one() {
+  static_assert(SmemLayout::total<MM>() <= 227 * 1024, "shared memory budget");
   return cudaFuncSetAttribute(k_stream<T, MM, Epi>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)SmemLayout::total<MM>());
 }

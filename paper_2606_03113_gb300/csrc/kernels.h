@@ -14,10 +14,10 @@ struct HeadPart {
   int32_t ti[kTopK];
 };
 
-// Exit-head statistics partials: one per 16-row vocabulary tile and one per
-// group of 64 tiles.
+// Per-block partial slots of the streamed kernels (running + split), for up
+// to kMaxBlocks blocks.
+constexpr int kMaxBlocks = 512;
 inline int head_tiles(int V) { return (V + 15) / 16; }
-inline int head_groups(int V) { return (head_tiles(V) + 63) / 64; }
 
 // big = true selects the kernels instantiated for up to kMaxM rows; false
 // the single-row ones.
