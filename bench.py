@@ -315,7 +315,7 @@ def main():
     if args.kernels_only:
         eng.set_ar()
         eng.prefill(ids)
-        roof = kernel_roofline(eng, w, peak, pos0=w.prompt_len, iters=2, graphs=False)
+        roof = kernel_roofline(eng, w, peak, pos0=w.prompt_len, iters=3, graphs=True)
         if rank == 0:
             print(json.dumps(dict(kernels=roof, workload=w.name, peak=peak)), flush=True)
         eng.close()

@@ -61,7 +61,7 @@ size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
   d.num_sms = kMaxBlocks;  // set to the device's SM count at init
   d.ss_tiles = (c.d_model + 15) / 16;
   d.max_tiles = std::max(
-      std::max(head_tiles(c.vocab), c.ffn_dim / 8 + 1),
+      std::max(head_tiles(c.vocab), c.ffn_dim / 16 + 1),
       std::max((c.n_heads + 2 * c.n_kv_heads) * c.head_dim / 16 + 2, c.d_model / 16 + 1));
   const size_t elt = c.dtype == SSD_DTYPE_BF16 ? 2 : 4;
   Carve cv{base};
@@ -71,7 +71,7 @@ size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
   b.ss = cv.take<float>(sizeof(float) * 2 * kMaxM);
   b.ss_tile = cv.take<float>(sizeof(float) * 2 * 2 * kMaxM * (size_t)kMaxBlocks);
   b.ss_counter = cv.take<uint32_t>(sizeof(uint32_t) * 2);
-  b.gpart = cv.take<float>(sizeof(float) * (size_t)kMaxBlocks * 2 * 16 * kMaxM);
+  b.gpart = cv.take<float>(sizeof(float) * (size_t)kMaxBlocks * 2 * 32 * kMaxM);
   b.tile_counter = cv.take<uint32_t>(sizeof(uint32_t) * (size_t)d.max_tiles);
 
   b.xq = cv.take<float>(sizeof(float) * kMaxM * d.qd);

@@ -5,19 +5,20 @@
 // rows (1 while drafting, k + 1 while verifying): at these M the work is bound
 // by HBM bandwidth.  Design (one kernel per matrix, persistent grid of one
 // block per SM):
-//  - the matrix is cut into stages of 16 rows x 2048 bytes; the stages, in
+//  - the matrix is cut into units of 32 rows x 512 bytes; the units, in
 //    (row tile, K) order, are split evenly over the blocks ("stream-K"), so
-//    every SM streams the same number of bytes whatever the matrix shape;
-//  - a producer warp copies each stage into a 6-deep shared-memory ring with
-//    1-D bulk async copies (one 2 KB copy per row: smaller copies starve the
-//    copy engine; evict-first in L2), synchronised by
+//    every SM streams the same number of bytes whatever the matrix shape, and
+//    a block copies up to four consecutive units of a tile as one stage;
+//  - a producer warp copies each stage into a 3-deep shared-memory ring with
+//    1-D bulk async copies (one copy of up to 2 KB per row: smaller copies
+//    starve the copy engine; evict-first in L2), synchronised by
 //    mbarriers; its copies do not wait for the previous kernel (programmatic
 //    dependent launch), so the weight stream of one kernel overlaps the tail
 //    of the previous one;
-//  - eight consumer warps read the stage from shared memory (two rows per
-//    warp, 16 bytes per lane per 512-byte step), multiply with the fp32 input
-//    rows (from L1/L2) and accumulate; a 16-row tile is reduced with warp
-//    shuffles;
+//  - eight consumer warps read the stage from shared memory (four rows per
+//    warp, so each input load serves four rows; 16 bytes per lane per
+//    512-byte step), multiply with the fp32 input rows (from L1/L2) and
+//    accumulate; a 32-row tile is reduced with warp shuffles;
 //  - a tile split between two blocks is finished by whichever block completes
 //    its share last (per-tile ticket), which adds the partial sums in block
 //    order, so results do not depend on scheduling;
@@ -34,24 +35,28 @@
 
 namespace ssd {
 
-constexpr int kRT = 16;             // rows per tile
-constexpr int kRowBytes = 2048;     // bytes of one row per stage
-constexpr int kNS = 6;              // ring depth
+constexpr int kRT = 32;             // rows per tile
+constexpr int kRowBytes = 2048;     // bytes of one row per stage (4 units)
+constexpr int kUnit = 512;          // bytes of one row per assignment unit
+constexpr int kNS = 3;              // ring depth
 constexpr int kCWarps = 8;          // consumer warps
 constexpr int kCThreads = kCWarps * 32;
 constexpr int kThreads = kCThreads + 32;  // + producer warp
-constexpr int kStageBytes = kRT * kRowBytes;
+constexpr int kRowStride = kRowBytes + 16;  // padded row pitch in shared memory:
+                                            // rows of an 8x8 ldmatrix land on distinct banks
+constexpr int kStageBytes = kRT * kRowStride;
+constexpr int kNB = (kMaxM + 7) / 8;        // 8-token column blocks of the tensor-core path
 constexpr int kMaxBlocksDev = 512;  // upper bound on the grid (partial slots per block)
 
 enum RowMap : int { kMapLinear = 0, kMapQKV = 1, kMapGateUp = 2 };
 
 struct Geom {
   int N, K;          // rows, columns (elements)
-  int nks;           // K steps per tile
+  int nks;           // 512-byte units per row (per tile)
   int ntiles;
-  long long T;       // stages
+  long long T;       // units (tiles x nks)
   int P;             // blocks
-  int last_bytes;    // bytes per row of the last K step
+  int row_bytes;     // K * elt
   int map;           // RowMap
   int elt;           // element size in bytes
 };
@@ -79,33 +84,33 @@ __device__ inline int block_of_stage(const Geom& g, long long s) {
   return b;
 }
 
-// Global row of local row r (0..15) of a tile, or -1 past the end.  QKV
-// tiles of a query/key head hold rows i..i+7 and their rotary partners
-// i+hd/2..i+hd/2+7; gate/up tiles hold gate rows j..j+7 and up rows F+j..F+j+7.
+// Global row of local row r (0..31) of a tile, or -1 past the end.  QKV
+// tiles of a query/key head hold rows i..i+15 and their rotary partners
+// i+hd/2..i+hd/2+15; gate/up tiles hold gate rows j..j+15 and up rows
+// F+j..F+j+15.
 __device__ inline int map_row(const Geom& g, const Dims& D, int tile, int r) {
   if (g.map == kMapQKV) {
-    const int tpp = D.hd / 16;             // tiles per query/key head
+    const int tpp = D.hd / 32;             // tiles per query/key head
     const int tqk = (D.Hq + D.Hkv) * tpp;
     if (tile < tqk) {
       const int h = tile / tpp, sub = tile - h * tpp;
-      return h * D.hd + (r < 8 ? sub * 8 + r : D.hd / 2 + sub * 8 + (r - 8));
+      return h * D.hd + (r < 16 ? sub * 16 + r : D.hd / 2 + sub * 16 + (r - 16));
     }
     const int row = (D.Hq + D.Hkv) * D.hd + (tile - tqk) * kRT + r;
     return row < g.N ? row : -1;
   }
   if (g.map == kMapGateUp) {
     const int F = g.N / 2;
-    const int j = tile * 8 + (r & 7);
+    const int j = tile * 16 + (r & 15);
     if (j >= F) return -1;
-    return r < 8 ? j : F + j;
+    return r < 16 ? j : F + j;
   }
   const int row = tile * kRT + r;
   return row < g.N ? row : -1;
 }
 
-// Local rows handled by consumer warp w: w and w + 8, the pairs the QKV and
-// gate/up epilogues combine.
-__device__ __forceinline__ int warp_row(int w, int i) { return w + 8 * i; }
+// Local rows handled by consumer warp w: w, w+8, w+16, w+24; (w, w+16) and
+// (w+8, w+24) are the pairs the QKV and gate/up epilogues combine.
 
 struct SmemLayout {
   static constexpr size_t ring = 0;
@@ -113,9 +118,11 @@ struct SmemLayout {
   static constexpr size_t rs = bars + 2 * kNS * sizeof(uint64_t);
   static constexpr size_t flag = rs + sizeof(float) * 32;
   static constexpr size_t scratch = flag + 64;  // cross-warp combine buffer
-  // combine buffers are indexed [warp][kMaxM] whatever MM is
+  static constexpr size_t red = scratch + (size_t)(kCWarps + 1) * kMaxM * sizeof(HeadPart);
   template <int MM>
-  static constexpr size_t total() { return scratch + (size_t)kCWarps * kMaxM * sizeof(HeadPart); }
+  static constexpr size_t total() {  // + tensor-core partial sums [4 K-quarters][32][8 kNB]
+    return red + sizeof(float) * 4 * kRT * 8 * kNB;
+  }
 };
 
 // Block b owns the exit-head / norm partial of the tile it starts and shares
@@ -156,9 +163,37 @@ __device__ inline void part_empty(HeadPart& p) {
   }
 }
 
-// a <- merge(a, b); symmetric in a and b (max, commutative sums, ordered
-// top-k), so both lanes of a shuffle exchange compute the same result.
+// Inserts (v, idx) into the descending top-k list with compare-swaps at fixed
+// positions (no runtime indexing, so the list stays in registers).
+__device__ __forceinline__ void topk_insert(float (&tv)[kTopK], int (&ti)[kTopK], float v, int idx) {
+#pragma unroll
+  for (int q = 0; q < kTopK; ++q) {
+    const bool b = better(v, idx, tv[q], ti[q]);
+    const float tvq = tv[q];
+    const int tiq = ti[q];
+    tv[q] = b ? v : tvq;
+    ti[q] = b ? idx : tiq;
+    v = b ? tvq : v;
+    idx = b ? tiq : idx;
+  }
+}
+
+__device__ __forceinline__ void cswap(float (&tv)[kTopK], int (&ti)[kTopK], int i, int j) {
+  const bool keep = better(tv[i], ti[i], tv[j], ti[j]);
+  const float a = tv[i], b = tv[j];
+  const int ia = ti[i], ib = ti[j];
+  tv[i] = keep ? a : b;
+  ti[i] = keep ? ia : ib;
+  tv[j] = keep ? b : a;
+  ti[j] = keep ? ib : ia;
+}
+
+// a <- merge(a, b); symmetric in a and b (max, commutative sums, a total
+// order on (value, index)), so both lanes of a shuffle exchange compute the
+// same result.  Top-k: bitonic merge of the two sorted lists (elementwise
+// best of a[i] and b[k-1-i], then a sorting network of 12 compare-swaps).
 __device__ inline void part_merge(HeadPart& a, const HeadPart& b) {
+  static_assert(kTopK == 8, "bitonic network written for 8");
   if (b.S > 0.f) {
     if (a.S > 0.f) {
       const float mx = fmaxf(a.mx, b.mx);
@@ -174,52 +209,37 @@ __device__ inline void part_merge(HeadPart& a, const HeadPart& b) {
       a.T = b.T;
     }
   }
-  float tv[kTopK];
-  int ti[kTopK];
-  int ia = 0, ib = 0;
 #pragma unroll
-  for (int q = 0; q < kTopK; ++q) {
-    const bool ta = better(a.tv[ia], a.ti[ia], b.tv[ib], b.ti[ib]);
-    tv[q] = ta ? a.tv[ia] : b.tv[ib];
-    ti[q] = ta ? a.ti[ia] : b.ti[ib];
-    ia += ta;
-    ib += !ta;
+  for (int i = 0; i < kTopK; ++i) {
+    const bool keep = better(a.tv[i], a.ti[i], b.tv[kTopK - 1 - i], b.ti[kTopK - 1 - i]);
+    a.tv[i] = keep ? a.tv[i] : b.tv[kTopK - 1 - i];
+    a.ti[i] = keep ? a.ti[i] : b.ti[kTopK - 1 - i];
   }
 #pragma unroll
-  for (int q = 0; q < kTopK; ++q) {
-    a.tv[q] = tv[q];
-    a.ti[q] = ti[q];
-  }
+  for (int i = 0; i < 4; ++i) cswap(a.tv, a.ti, i, i + 4);
+  cswap(a.tv, a.ti, 0, 2);
+  cswap(a.tv, a.ti, 1, 3);
+  cswap(a.tv, a.ti, 4, 6);
+  cswap(a.tv, a.ti, 5, 7);
+#pragma unroll
+  for (int i = 0; i < 8; i += 2) cswap(a.tv, a.ti, i, i + 1);
 }
 
 // Adds one logit z of vocabulary row idx.
 __device__ inline void part_add(HeadPart& p, float z, int idx) {
   if (!(z > -INFINITY)) return;
   if (p.S > 0.f) {
-    if (z > p.mx) {
-      const float e = expf(p.mx - z);
-      p.T = e * (p.T + (p.mx - z) * p.S);
-      p.S = p.S * e + 1.f;
-      p.mx = z;
-    } else {
-      const float e = expf(z - p.mx);
-      p.S += e;
-      p.T += e * (z - p.mx);
-    }
+    const float mx = fmaxf(p.mx, z);
+    const float e_old = expf(p.mx - mx), e_new = expf(z - mx);
+    p.T = e_old * (p.T + (p.mx - mx) * p.S) + e_new * (z - mx);
+    p.S = p.S * e_old + e_new;
+    p.mx = mx;
   } else {
     p.mx = z;
     p.S = 1.f;
     p.T = 0.f;
   }
-  if (!better(z, idx, p.tv[kTopK - 1], p.ti[kTopK - 1])) return;
-  int q = kTopK - 1;
-  while (q > 0 && better(z, idx, p.tv[q - 1], p.ti[q - 1])) {
-    p.tv[q] = p.tv[q - 1];
-    p.ti[q] = p.ti[q - 1];
-    --q;
-  }
-  p.tv[q] = z;
-  p.ti[q] = idx;
+  topk_insert(p.tv, p.ti, z, idx);
 }
 
 __device__ inline HeadPart part_shfl(const HeadPart& p, int off) {
@@ -257,7 +277,7 @@ struct EpiPlain {
   __device__ void init(State&) const {}
   __device__ void pair(const StreamArgs& a, int tile, int w, int m, int, float, float v0, float v1,
                        State&) const {
-    const int r0 = map_row(a.g, a.D, tile, w), r1 = map_row(a.g, a.D, tile, w + 8);
+    const int r0 = map_row(a.g, a.D, tile, w), r1 = map_row(a.g, a.D, tile, w + 16);
     if (r0 >= 0) y[(size_t)m * a.g.N + r0] = v0;
     if (r1 >= 0) y[(size_t)m * a.g.N + r1] = v1;
   }
@@ -276,7 +296,7 @@ struct EpiQKV {
   __device__ void pair(const StreamArgs& a, int tile, int w, int m, int pos0, float rs, float v0,
                        float v1, State&) const {
     const Dims& D = a.D;
-    const int tqk = (D.Hq + D.Hkv) * (D.hd / 16);
+    const int tqk = (D.Hq + D.Hkv) * (D.hd / 32);
     T* kv = static_cast<T*>(a.B.kv) + (size_t)layer * 2 * D.Hkv * D.max_seq * D.hd;
     const int pos = pos0 + m;
     const float y0 = v0 * rs, y1 = v1 * rs;
@@ -297,7 +317,7 @@ struct EpiQKV {
         kr[i + half] = Elem<T>::from_f(o1);
       }
     } else {
-      const int r1 = map_row(a.g, D, tile, w + 8);
+      const int r1 = map_row(a.g, D, tile, w + 16);
       const int vb = (D.Hq + D.Hkv) * D.hd;
       if (r0 >= 0) {
         const int g = (r0 - vb) / D.hd, j = (r0 - vb) - g * D.hd;
@@ -353,7 +373,7 @@ struct EpiResid {
   __device__ void init(State& s) const { s.ss = 0.f; }
   __device__ void pair(const StreamArgs& a, int tile, int w, int m, int, float, float v0, float v1,
                        State& st) const {
-    const int r0 = map_row(a.g, a.D, tile, w), r1 = map_row(a.g, a.D, tile, w + 8);
+    const int r0 = map_row(a.g, a.D, tile, w), r1 = map_row(a.g, a.D, tile, w + 16);
     float* hm = a.B.h + (size_t)m * a.D.d;
     if (r0 >= 0) {
       const float h = hm[r0] + v0;
@@ -384,33 +404,47 @@ struct EpiResid {
     named_sync(1, kCThreads);
     if (!*sh.flag) return;
     __threadfence();
+    // every thread loads its slots first, then a fixed reduction tree
+    float* buf = static_cast<float*>(sh.scratch);
     const int warp = tid >> 5, lane = tid & 31;
-    for (int m = warp; m < M; m += kCWarps) {
+    for (int m = 0; m < M; ++m) {
       float v = 0.f;
-      for (int b = lane; b < a.g.P; b += 32) {
+      for (int b = tid; b < a.g.P; b += kCThreads) {
         v += __ldcg(&sl[(size_t)b * kMaxM + m]);
         if (has_split_slot(a.g, b)) v += __ldcg(&sl[((size_t)kMaxBlocksDev + b) * kMaxM + m]);
       }
       v = warp_sum(v);
-      if (lane == 0) a.B.ss[which * kMaxM + m] = v;
+      if (lane == 0) buf[warp] = v;
+      named_sync(1, kCThreads);
+      if (tid == 0) {
+        float t = 0.f;
+        for (int w = 0; w < kCWarps; ++w) t += buf[w];
+        a.B.ss[which * kMaxM + m] = t;
+      }
+      named_sync(1, kCThreads);
     }
     if (tid == 0) a.B.ss_counter[which] = 0u;
   }
 };
 
-// Merges the per-lane statistics of the 8 warps (lane m of each) in warp
-// order; result in thread m < M.
-__device__ inline HeadPart combine_parts(const HeadPart& p, const Shared& sh, int tid, int M) {
+// Merges the per-lane statistics of the 8 warps (lane m of each) with a
+// fixed shuffle tree and leaves row m's result in out[m] (shared memory).
+__device__ inline void combine_parts(const HeadPart& p, const Shared& sh, int tid, int M,
+                                     HeadPart* out) {
   HeadPart* buf = static_cast<HeadPart*>(sh.scratch);
   const int warp = tid >> 5, lane = tid & 31;
   if (lane < M) buf[warp * kMaxM + lane] = p;
   named_sync(1, kCThreads);
-  HeadPart r;
-  part_empty(r);
-  if (tid < M)
-    for (int w = 0; w < kCWarps; ++w) part_merge(r, buf[w * kMaxM + tid]);
+  for (int m = warp; m < M; m += kCWarps) {
+    HeadPart q;
+    if (lane < kCWarps)
+      q = buf[lane * kMaxM + m];
+    else
+      part_empty(q);
+    for (int off = 4; off > 0; off >>= 1) part_merge(q, part_shfl(q, off));
+    if (lane == 0) out[m] = q;
+  }
   named_sync(1, kCThreads);
-  return r;
 }
 
 // Exit head: z = W_lm RMSNorm_final(h).  Lane m keeps running statistics of
@@ -427,7 +461,7 @@ struct EpiHead {
   __device__ void init(State& s) const { part_empty(s.p); }
   __device__ void pair(const StreamArgs& a, int tile, int w, int m, int, float rs, float v0,
                        float v1, State& st) const {
-    const int r0 = map_row(a.g, a.D, tile, w), r1 = map_row(a.g, a.D, tile, w + 8);
+    const int r0 = map_row(a.g, a.D, tile, w), r1 = map_row(a.g, a.D, tile, w + 16);
     if (r0 >= 0) {
       const float z = v0 * rs;
       part_add(st.p, z, r0);
@@ -444,45 +478,62 @@ struct EpiHead {
   }
   __device__ void split_done(const StreamArgs& a, int b0, State& st, const Shared& sh, int tid,
                              int M) const {
-    const HeadPart r = combine_parts(st.p, sh, tid, M);
-    if (tid < M) slots(a)[((size_t)kMaxBlocksDev + b0) * kMaxM + tid] = r;
+    HeadPart* out = static_cast<HeadPart*>(sh.scratch) + kCWarps * kMaxM;
+    combine_parts(st.p, sh, tid, M, out);
+    if (tid < M) slots(a)[((size_t)kMaxBlocksDev + b0) * kMaxM + tid] = out[tid];
   }
   __device__ void finish(const StreamArgs& a, State& st, const Shared& sh, int tid, int M) const {
-    const HeadPart r = combine_parts(st.p, sh, tid, M);
+    HeadPart* out = static_cast<HeadPart*>(sh.scratch) + kCWarps * kMaxM;
+    combine_parts(st.p, sh, tid, M, out);
     HeadPart* sl = slots(a);
-    if (tid < M) sl[(size_t)blockIdx.x * kMaxM + tid] = r;
+    if (tid < M) sl[(size_t)blockIdx.x * kMaxM + tid] = out[tid];
     __threadfence();
     named_sync(1, kCThreads);
     if (tid == 0) *sh.flag = atomicAdd(a.B.head_counter, 1u) == (unsigned)(a.g.P - 1);
     named_sync(1, kCThreads);
     if (!*sh.flag) return;
     __threadfence();
+    // every thread merges its slots, then a fixed shuffle tree per warp and
+    // one over the eight warp results
+    HeadPart* buf = static_cast<HeadPart*>(sh.scratch);
     const int warp = tid >> 5, lane = tid & 31;
-    for (int m = warp; m < M; m += kCWarps) {
+    for (int m = 0; m < M; ++m) {
       HeadPart p;
       part_empty(p);
-      for (int b = lane; b < a.g.P; b += 32) {
+      for (int b = tid; b < a.g.P; b += kCThreads) {
         part_merge(p, part_load_cg(&sl[(size_t)b * kMaxM + m]));
         if (has_split_slot(a.g, b)) part_merge(p, part_load_cg(&sl[((size_t)kMaxBlocksDev + b) * kMaxM + m]));
       }
       for (int off = 16; off > 0; off >>= 1) part_merge(p, part_shfl(p, off));
-      if (lane == 0) {
-        RowStats& o = a.B.stats[m];
-        const float logS = logf(p.S);
-        o.argmax = p.ti[0];
-        o.zmax = p.mx;
-        o.lse = p.mx + logS;
-        o.entropy = logS - p.T / p.S;
-        float tsum = 0.f;
-        for (int q = 0; q < kTopK; ++q) {
-          o.top_idx[q] = p.ti[q];
-          o.top_logit[q] = p.tv[q];
-          if (q < topk) tsum += p.tv[q];
+      if (lane == 0) buf[warp] = p;
+      named_sync(1, kCThreads);
+      if (warp == 0) {
+        HeadPart f;
+        if (lane < kCWarps)
+          f = buf[lane];
+        else
+          part_empty(f);
+        for (int off = 4; off > 0; off >>= 1) part_merge(f, part_shfl(f, off));
+        if (lane == 0) {
+          RowStats& o = a.B.stats[m];
+          const float logS = logf(f.S);
+          o.argmax = f.ti[0];
+          o.zmax = f.mx;
+          o.lse = f.mx + logS;
+          o.entropy = logS - f.T / f.S;
+          float tsum = 0.f;
+#pragma unroll
+          for (int q = 0; q < kTopK; ++q) {
+            o.top_idx[q] = f.ti[q];
+            o.top_logit[q] = f.tv[q];
+            if (q < topk) tsum += f.tv[q];
+          }
+          o.conf_k = o.lse - tsum / (float)topk;
+          o.pmax = 1.0f / f.S;
+          o.margin = f.tv[0] - f.tv[1];
         }
-        o.conf_k = o.lse - tsum / (float)topk;
-        o.pmax = 1.0f / p.S;
-        o.margin = p.tv[0] - p.tv[1];
       }
+      named_sync(1, kCThreads);
     }
     if (tid == 0) *a.B.head_counter = 0u;
   }
@@ -499,11 +550,53 @@ __device__ __forceinline__ float pick(const float (&v)[MM], int lane) {
   return r;
 }
 
-template <typename T, int MM, class Epi>
+// ---- tensor-core helpers (verification rows: M > 1)
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& a0, uint32_t& a1, uint32_t& a2,
+                                        uint32_t& a3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(a0), "=r"(a1), "=r"(a2), "=r"(a3)
+               : "r"(addr));
+}
+
+// d += A(16x16, bf16, row) * B(16x8, bf16, col), fp32 accumulate.
+__device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                          uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Splits (x0, x1) into bf16 high parts and bf16 residuals, packed low-k first:
+// x = hi + lo to about 16 significant bits, so two bf16 products keep the
+// activations' fp32 precision.
+__device__ __forceinline__ void split_bf16x2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
+  const __nv_bfloat16 l0 = __float2bfloat16_rn(x0 - __bfloat162float(h0));
+  const __nv_bfloat16 l1 = __float2bfloat16_rn(x1 - __bfloat162float(h1));
+  hi = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+  lo = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+}
+
+// Stage sequence of a block: from unit u, the run of up to 4 units that stays
+// inside the tile and the block's range.  Producer and consumers walk it
+// identically.
+__device__ __forceinline__ int stage_units(const Geom& g, long long u, long long u_end) {
+  const long long j = u % g.nks;
+  long long n = g.nks - j;
+  if (n > kRowBytes / kUnit) n = kRowBytes / kUnit;
+  if (n > u_end - u) n = u_end - u;
+  return (int)n;
+}
+
+template <typename T, int MM, bool NORM, bool MMA, class Epi>
 __global__ void __launch_bounds__(kThreads, 1) k_stream(const StreamArgs a, const Epi epi) {
+  static_assert(!MMA || (std::is_same<T, __nv_bfloat16>::value && MM > 1), "tensor path: bf16 rows");
   extern __shared__ __align__(128) unsigned char smem[];
   using E = Elem<T>;
   constexpr int EPC = E::kPerChunk;
+  constexpr int CU = kUnit / (int)sizeof(T);  // columns per unit
   unsigned char* ring = smem + SmemLayout::ring;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + SmemLayout::bars);
   uint64_t* empty = full + kNS;
@@ -512,7 +605,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_stream(const StreamArgs a, cons
 
   const Geom& g = a.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long long s_begin = stage_start(g, blockIdx.x), s_end = stage_start(g, blockIdx.x + 1);
+  const long long u_begin = stage_start(g, blockIdx.x), u_end = stage_start(g, blockIdx.x + 1);
   if (threadIdx.x == 0) {
     for (int i = 0; i < kNS; ++i) {
       mbar_init(&full[i], 1);
@@ -527,29 +620,30 @@ __global__ void __launch_bounds__(kThreads, 1) k_stream(const StreamArgs a, cons
     // ---------------- producer: weights do not depend on earlier kernels
     const unsigned char* W = static_cast<const unsigned char*>(a.W);
     const uint64_t pol = evict_first_policy();
-    long long issued = 0;
-    for (long long s = s_begin; s < s_end; ++s, ++issued) {
-      const int i = (int)(s - s_begin), slot = i % kNS;
+    int i = 0;
+    for (long long u = u_begin; u < u_end; ++i) {
+      const int n = stage_units(g, u, u_end);
+      const int slot = i % kNS;
       const uint32_t ph = (uint32_t)(i / kNS) & 1u;
       if (!mbar_wait(&empty[slot], ph ^ 1u)) {
         if (lane == 0) atomicOr(&a.B.ctl->err, (int)kErrTimeout);
         break;
       }
-      const int tile = (int)(s / g.nks), ks = (int)(s - (long long)tile * g.nks);
-      const int rb = ks == g.nks - 1 ? g.last_bytes : kRowBytes;
-      const int row = lane < kRT ? map_row(g, a.D, tile, lane) : -1;
+      const int tile = (int)(u / g.nks), j = (int)(u - (long long)tile * g.nks);
+      const int off = j * kUnit;
+      const int bytes = min(n * kUnit, g.row_bytes - off);
+      const int row = map_row(g, a.D, tile, lane);
       const int nvalid = __popc(__ballot_sync(0xffffffffu, row >= 0));
-      if (lane == 0) mbar_arrive_expect_tx(&full[slot], (uint32_t)(nvalid * rb));
+      if (lane == 0) mbar_arrive_expect_tx(&full[slot], (uint32_t)(nvalid * bytes));
       __syncwarp();
       if (row >= 0)
-        bulk_g2s(ring + (size_t)slot * kStageBytes + lane * kRowBytes,
-                 W + ((size_t)row * g.K) * g.elt + (size_t)ks * kRowBytes, (uint32_t)rb,
-                 &full[slot], pol);
+        bulk_g2s(ring + (size_t)slot * kStageBytes + lane * kRowStride,
+                 W + (size_t)row * g.row_bytes + off, (uint32_t)bytes, &full[slot], pol);
+      u += n;
     }
     // drain: the copies of the last stages have landed before the block exits
     if (lane == 0)
-      for (long long i = issued > kNS ? issued - kNS : 0; i < issued; ++i)
-        mbar_wait(&full[i % kNS], (uint32_t)(i / kNS) & 1u);
+      for (int k = i > kNS ? i - kNS : 0; k < i; ++k) mbar_wait(&full[k % kNS], (uint32_t)(k / kNS) & 1u);
     return;
   }
 
@@ -566,90 +660,226 @@ __global__ void __launch_bounds__(kThreads, 1) k_stream(const StreamArgs a, cons
   named_sync(1, kCThreads);
   const float my_rs = sh.rs[lane];
   const float* x = a.x;
-  const T* gn = static_cast<const T*>(a.gnorm);
-  const int KC = kRowBytes / (int)sizeof(T);
+  const T* gn = static_cast<const T*>(a.gnorm);  // used when NORM
   typename Epi::State run;
   epi.init(run);
-  float acc[2][MM];
-  const int rloc[2] = {warp, warp + 8};
+  float acc[MMA ? 1 : 4][MMA ? 1 : MM];
+  float dmm[kNB][4];  // tensor-core accumulators: rows rb*16 + (g, g+8), tokens nb*8 + 2c + (0, 1)
+  float* red = reinterpret_cast<float*>(smem + SmemLayout::red);
+  const int rloc[4] = {warp, warp + 8, warp + 16, warp + 24};
   int cur = -1;
   bool ok = true;
-  for (long long s = s_begin; s < s_end; ++s) {
-    const int i = (int)(s - s_begin), slot = i % kNS;
+  int i = 0;
+  for (long long u = u_begin; u < u_end; ++i) {
+    const int n = stage_units(g, u, u_end);
+    const int slot = i % kNS;
     const uint32_t ph = (uint32_t)(i / kNS) & 1u;
-    const int tile = (int)(s / g.nks), ks = (int)(s - (long long)tile * g.nks);
+    const int tile = (int)(u / g.nks), j = (int)(u - (long long)tile * g.nks);
+    u += n;
     if (tile != cur) {
+      if (MMA) {
 #pragma unroll
-      for (int r = 0; r < 2; ++r)
+        for (int nb = 0; nb < kNB; ++nb)
 #pragma unroll
-        for (int m = 0; m < MM; ++m) acc[r][m] = 0.f;
+          for (int q = 0; q < 4; ++q) dmm[nb][q] = 0.f;
+      } else {
+#pragma unroll
+        for (int r = 0; r < (MMA ? 1 : 4); ++r)
+#pragma unroll
+          for (int m = 0; m < (MMA ? 1 : MM); ++m) acc[r][m] = 0.f;
+      }
       cur = tile;
     }
     if (ok && !mbar_wait(&full[slot], ph)) {
       if (lane == 0) atomicOr(&a.B.ctl->err, (int)kErrTimeout);
       ok = false;
     }
-    const int rb = ks == g.nks - 1 ? g.last_bytes : kRowBytes;
-#pragma unroll
-    for (int sub = 0; sub < kRowBytes / 512; ++sub) {
-      const int off = sub * 512 + lane * 16;
-      if (!ok || off >= rb) break;
-      const unsigned char* st = ring + (size_t)slot * kStageBytes + off;
-      float wf[2][EPC];
-#pragma unroll
-      for (int r = 0; r < 2; ++r)
-        E::unpack(*reinterpret_cast<const uint4*>(st + rloc[r] * kRowBytes), wf[r]);
-      const int col = ks * KC + off / (int)sizeof(T);
-      float gv[EPC];
-      if (gn) {
-        E::unpack(__ldg(reinterpret_cast<const uint4*>(gn + col)), gv);
-      } else {
-#pragma unroll
-        for (int e = 0; e < EPC; ++e) gv[e] = 1.f;
-      }
-#pragma unroll
-      for (int m = 0; m < MM; ++m) {
-        if (m < M) {
-          float xv[EPC];
-          const float4* xp = reinterpret_cast<const float4*>(x + (size_t)m * g.K + col);
-#pragma unroll
-          for (int q = 0; q < EPC / 4; ++q) {
-            const float4 t4 = __ldg(xp + q);
-            xv[4 * q] = t4.x * gv[4 * q];
-            xv[4 * q + 1] = t4.y * gv[4 * q + 1];
-            xv[4 * q + 2] = t4.z * gv[4 * q + 2];
-            xv[4 * q + 3] = t4.w * gv[4 * q + 3];
+    const int bytes = min(n * kUnit, g.row_bytes - j * kUnit);
+    const unsigned char* stg = ring + (size_t)slot * kStageBytes + lane * 16;
+    const int col0 = j * CU + lane * 16 / (int)sizeof(T);
+    if constexpr (MMA) {
+      // warp = (16-row block rb, 512-byte unit kq of the stage)
+      const int rb = warp & 1, kq = warp >> 1;
+      if (ok && kq < n) {
+        const int ub = min(kUnit, bytes - kq * kUnit);
+        const uint32_t abase =
+            smem_u32(ring + (size_t)slot * kStageBytes + (rb * 16 + (lane & 15)) * kRowStride +
+                     kq * kUnit + (lane >> 4) * 16);
+        const int kc0 = (j + kq) * CU + 2 * (lane & 3);
+        const int tok0 = lane >> 2;
+        for (int kk = 0; kk < ub / 32; ++kk) {
+          uint32_t a0, a1, a2, a3;
+          ldsm_x4(abase + kk * 32, a0, a1, a2, a3);
+          const int kc = kc0 + kk * 16;
+          float g0 = 1.f, g1 = 1.f, g8 = 1.f, g9 = 1.f;
+          if (NORM) {
+            const __nv_bfloat162 ga = *reinterpret_cast<const __nv_bfloat162*>(gn + kc);
+            const __nv_bfloat162 gb = *reinterpret_cast<const __nv_bfloat162*>(gn + kc + 8);
+            g0 = __low2float(ga);
+            g1 = __high2float(ga);
+            g8 = __low2float(gb);
+            g9 = __high2float(gb);
           }
 #pragma unroll
-          for (int r = 0; r < 2; ++r)
+          for (int nb = 0; nb < kNB; ++nb) {
+            if (nb * 8 < M) {
+              const int tok = nb * 8 + tok0;
+              float2 xa = make_float2(0.f, 0.f), xb = make_float2(0.f, 0.f);
+              if (tok < M) {
+                xa = __ldg(reinterpret_cast<const float2*>(x + (size_t)tok * g.K + kc));
+                xb = __ldg(reinterpret_cast<const float2*>(x + (size_t)tok * g.K + kc + 8));
+              }
+              uint32_t h0, l0, h1, l1;
+              split_bf16x2(xa.x * g0, xa.y * g1, h0, l0);
+              split_bf16x2(xb.x * g8, xb.y * g9, h1, l1);
+              mma_16816(dmm[nb], a0, a1, a2, a3, h0, h1);
+              mma_16816(dmm[nb], a0, a1, a2, a3, l0, l1);
+            }
+          }
+        }
+      }
+    } else if (ok && bytes == kRowBytes) {
+      // full stage; the single-row kernel issues every load of the stage
+      // before the math, the multi-row one goes one 512-byte step at a time
+      constexpr int NSUB = kRowBytes / kUnit;
+      constexpr int HOIST = MM <= 2 ? NSUB : 1;
 #pragma unroll
-            for (int e = 0; e < EPC; ++e) acc[r][m] = fmaf(wf[r][e], xv[e], acc[r][m]);
+      for (int sg = 0; sg < NSUB; sg += HOIST) {
+        uint4 wq[HOIST][4];
+#pragma unroll
+        for (int h = 0; h < HOIST; ++h)
+#pragma unroll
+          for (int r = 0; r < 4; ++r)
+            wq[h][r] = *reinterpret_cast<const uint4*>(stg + rloc[r] * kRowStride + (sg + h) * kUnit);
+        float gv[HOIST][EPC];
+        if (NORM) {
+          uint4 gq[HOIST];
+#pragma unroll
+          for (int h = 0; h < HOIST; ++h)
+            gq[h] = __ldg(reinterpret_cast<const uint4*>(gn + col0 + (sg + h) * CU));
+#pragma unroll
+          for (int h = 0; h < HOIST; ++h) E::unpack(gq[h], gv[h]);
+        }
+#pragma unroll
+        for (int m = 0; m < MM; ++m) {
+          if (m < M) {
+            float4 xq[HOIST][EPC / 4];
+#pragma unroll
+            for (int h = 0; h < HOIST; ++h)
+#pragma unroll
+              for (int q = 0; q < EPC / 4; ++q)
+                xq[h][q] = __ldg(reinterpret_cast<const float4*>(x + (size_t)m * g.K + col0 +
+                                                                 (sg + h) * CU) + q);
+#pragma unroll
+            for (int h = 0; h < HOIST; ++h) {
+              float xv[EPC];
+#pragma unroll
+              for (int q = 0; q < EPC / 4; ++q) {
+                xv[4 * q] = xq[h][q].x;
+                xv[4 * q + 1] = xq[h][q].y;
+                xv[4 * q + 2] = xq[h][q].z;
+                xv[4 * q + 3] = xq[h][q].w;
+              }
+              if (NORM) {
+#pragma unroll
+                for (int e = 0; e < EPC; ++e) xv[e] *= gv[h][e];
+              }
+#pragma unroll
+              for (int r = 0; r < 4; ++r) {
+                float wf[EPC];
+                E::unpack(wq[h][r], wf);
+#pragma unroll
+                for (int e = 0; e < EPC; ++e) acc[r][m] = fmaf(wf[e], xv[e], acc[r][m]);
+              }
+            }
+          }
+        }
+      }
+    } else if (ok) {
+      // partial stage (block range edge or ragged end of the row)
+      for (int off = lane * 16; off < bytes; off += kUnit) {
+        const int col = j * CU + off / (int)sizeof(T);
+        float gv[EPC];
+        if (NORM) E::unpack(__ldg(reinterpret_cast<const uint4*>(gn + col)), gv);
+        float wf[4][EPC];
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+          E::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)slot * kStageBytes +
+                                                    rloc[r] * kRowStride + off), wf[r]);
+#pragma unroll
+        for (int m = 0; m < MM; ++m) {
+          if (m < M) {
+            float xv[EPC];
+            const float4* xp = reinterpret_cast<const float4*>(x + (size_t)m * g.K + col);
+#pragma unroll
+            for (int q = 0; q < EPC / 4; ++q) {
+              const float4 t4 = __ldg(xp + q);
+              xv[4 * q] = t4.x;
+              xv[4 * q + 1] = t4.y;
+              xv[4 * q + 2] = t4.z;
+              xv[4 * q + 3] = t4.w;
+            }
+            if (NORM) {
+#pragma unroll
+              for (int e = 0; e < EPC; ++e) xv[e] *= gv[e];
+            }
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+#pragma unroll
+              for (int e = 0; e < EPC; ++e) acc[r][m] = fmaf(wf[r][e], xv[e], acc[r][m]);
+          }
         }
       }
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(&empty[slot]);
-    if (ks != g.nks - 1 && s != s_end - 1) continue;
+    if (j + n != g.nks && u != u_end) continue;
 
     // ---- tile flush: warp-local unless the tile is shared with other blocks
-    float v[2][MM];
+    float val[4];  // lane m: the four rows' sums for input row m
+    if constexpr (MMA) {
+      // four K-quarter partials per row, added in quarter order
+      named_sync(1, kCThreads);
+      const int rb = warp & 1, kq = warp >> 1, gq = lane >> 2, cq = lane & 3;
 #pragma unroll
-    for (int r = 0; r < 2; ++r)
+      for (int nb = 0; nb < kNB; ++nb)
 #pragma unroll
-      for (int m = 0; m < MM; ++m) v[r][m] = m < M ? warp_sum(acc[r][m]) : 0.f;
+        for (int q = 0; q < 4; ++q) {
+          const int row = rb * 16 + gq + (q >> 1) * 8, tok = nb * 8 + 2 * cq + (q & 1);
+          red[((kq * kRT) + row) * 8 * kNB + tok] = dmm[nb][q];
+        }
+      named_sync(1, kCThreads);
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        float t = 0.f;
+        if (lane < M)
+          for (int q = 0; q < 4; ++q) t += red[((q * kRT) + rloc[r]) * 8 * kNB + lane];
+        val[r] = t;
+      }
+    } else {
+#pragma unroll
+      for (int r = 0; r < (MMA ? 1 : 4); ++r)
+#pragma unroll
+        for (int m = 0; m < (MMA ? 1 : MM); ++m)
+          if (m < M) acc[r][m] = warp_sum(acc[r][m]);
+#pragma unroll
+      for (int r = 0; r < (MMA ? 1 : 4); ++r) val[r] = pick(acc[r], lane);
+    }
     const long long t0 = (long long)tile * g.nks, t1 = t0 + g.nks;
-    if (t0 >= s_begin && t1 <= s_end) {
-      if (lane < M) epi.pair(a, tile, warp, lane, pos0, my_rs, pick(v[0], lane), pick(v[1], lane), run);
+    if (t0 >= u_begin && t1 <= u_end) {
+      if (lane < M) {
+        epi.pair(a, tile, warp, lane, pos0, my_rs, val[0], val[2], run);
+        epi.pair(a, tile, warp + 8, lane, pos0, my_rs, val[1], val[3], run);
+      }
       continue;
     }
     // shared with neighbouring blocks: publish this block's partial sums
-    const int first_tile = (int)(s_begin / g.nks);
+    const int first_tile = (int)(u_begin / g.nks);
     const int slot2 = tile == first_tile ? 0 : 1;
     float* mine = a.B.gpart + ((size_t)blockIdx.x * 2 + slot2) * kRT * kMaxM;
-    if (lane < M) {
-      mine[rloc[0] * kMaxM + lane] = pick(v[0], lane);
-      mine[rloc[1] * kMaxM + lane] = pick(v[1], lane);
-    }
+    if (lane < M)
+#pragma unroll
+      for (int r = 0; r < 4; ++r) mine[rloc[r] * kMaxM + lane] = val[r];
     __threadfence();
     named_sync(1, kCThreads);
     const int b0 = block_of_stage(g, t0), b1 = block_of_stage(g, t1 - 1);
@@ -661,20 +891,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_stream(const StreamArgs a, cons
     named_sync(1, kCThreads);
     if (!*sh.flag) continue;
     __threadfence();
-    float u0 = 0.f, u1 = 0.f;
+    float uu[4] = {0.f, 0.f, 0.f, 0.f};
     if (lane < M)
       for (int b = b0; b <= b1; ++b) {  // block order: independent of who finishes
         const long long sb = stage_start(g, b);
         if (sb == stage_start(g, b + 1)) continue;
         const int sl = tile == (int)(sb / g.nks) ? 0 : 1;
         const float* p = a.B.gpart + ((size_t)b * 2 + sl) * kRT * kMaxM;
-        u0 += __ldcg(&p[rloc[0] * kMaxM + lane]);
-        u1 += __ldcg(&p[rloc[1] * kMaxM + lane]);
+#pragma unroll
+        for (int r = 0; r < 4; ++r) uu[r] += __ldcg(&p[rloc[r] * kMaxM + lane]);
       }
     if (tid == 0) a.B.tile_counter[tile] = 0u;
     typename Epi::State sp;
     epi.init(sp);
-    if (lane < M) epi.pair(a, tile, warp, lane, pos0, my_rs, u0, u1, sp);
+    if (lane < M) {
+      epi.pair(a, tile, warp, lane, pos0, my_rs, uu[0], uu[2], sp);
+      epi.pair(a, tile, warp + 8, lane, pos0, my_rs, uu[1], uu[3], sp);
+    }
     epi.split_done(a, b0, sp, sh, tid, M);
   }
   epi.finish(a, run, sh, tid, M);
@@ -691,13 +924,12 @@ static Geom make_geom(const Dims& D, int N, int K, int elt, int map) {
   g.K = K;
   g.elt = elt;
   g.map = map;
-  const long long row_bytes = (long long)K * elt;
-  g.nks = (int)((row_bytes + kRowBytes - 1) / kRowBytes);
-  g.last_bytes = (int)(row_bytes - (long long)(g.nks - 1) * kRowBytes);
+  g.row_bytes = K * elt;
+  g.nks = (g.row_bytes + kUnit - 1) / kUnit;
   if (map == kMapGateUp)
-    g.ntiles = (N / 2 + 7) / 8;
+    g.ntiles = (N / 2 + 15) / 16;
   else if (map == kMapQKV)
-    g.ntiles = (D.Hq + D.Hkv) * (D.hd / 16) + (D.Hkv * D.hd + kRT - 1) / kRT;
+    g.ntiles = (D.Hq + D.Hkv) * (D.hd / 32) + (D.Hkv * D.hd + kRT - 1) / kRT;
   else
     g.ntiles = (N + kRT - 1) / kRT;
   g.T = (long long)g.ntiles * g.nks;
@@ -705,27 +937,44 @@ static Geom make_geom(const Dims& D, int N, int K, int elt, int map) {
   return g;
 }
 
-template <typename T, int MM, class Epi>
-static cudaError_t stream_launch(const StreamArgs& a, const Epi& epi, cudaStream_t st) {
-  return launch_ex(k_stream<T, MM, Epi>, dim3(a.g.P), dim3(kThreads), SmemLayout::total<MM>(), st,
-                   a, epi);
+// Multi-row bf16 matrices whose rows are whole 512-byte units go through the
+// tensor cores; single rows, fp32 and ragged rows through CUDA cores.
+template <typename T, int MM>
+static bool use_mma(const Geom& g) {
+  return std::is_same<T, __nv_bfloat16>::value && MM > 1 && g.row_bytes % kUnit == 0;
 }
 
-template <typename T, int MM, class Epi>
+template <typename T, int MM, bool NORM, class Epi>
+static cudaError_t stream_launch(const StreamArgs& a, const Epi& epi, cudaStream_t st) {
+  constexpr bool kCan = std::is_same<T, __nv_bfloat16>::value && MM > 1;
+  if (kCan && use_mma<T, MM>(a.g))
+    return launch_ex(k_stream<T, MM, NORM, kCan, Epi>, dim3(a.g.P), dim3(kThreads),
+                     SmemLayout::total<MM>(), st, a, epi);
+  return launch_ex(k_stream<T, MM, NORM, false, Epi>, dim3(a.g.P), dim3(kThreads),
+                   SmemLayout::total<MM>(), st, a, epi);
+}
+
+template <typename T, int MM, bool NORM, class Epi>
 static cudaError_t prepare_one() {
   static_assert(SmemLayout::total<MM>() <= 227 * 1024, "shared memory budget");
-  return cudaFuncSetAttribute(k_stream<T, MM, Epi>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  constexpr bool kCan = std::is_same<T, __nv_bfloat16>::value && MM > 1;
+  cudaError_t e = cudaFuncSetAttribute(k_stream<T, MM, NORM, false, Epi>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)SmemLayout::total<MM>());
+  if (e != cudaSuccess || !kCan) return e;
+  return cudaFuncSetAttribute(k_stream<T, MM, NORM, kCan, Epi>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)SmemLayout::total<MM>());
 }
 
 template <typename T, int MM>
 static cudaError_t prepare_t() {
   cudaError_t e;
-  if ((e = prepare_one<T, MM, EpiPlain>()) != cudaSuccess) return e;
-  if ((e = prepare_one<T, MM, EpiQKV<T>>()) != cudaSuccess) return e;
-  if ((e = prepare_one<T, MM, EpiGateUp>()) != cudaSuccess) return e;
-  if ((e = prepare_one<T, MM, EpiResid>()) != cudaSuccess) return e;
-  return prepare_one<T, MM, EpiHead>();
+  if ((e = prepare_one<T, MM, false, EpiPlain>()) != cudaSuccess) return e;
+  if ((e = prepare_one<T, MM, true, EpiQKV<T>>()) != cudaSuccess) return e;
+  if ((e = prepare_one<T, MM, true, EpiGateUp>()) != cudaSuccess) return e;
+  if ((e = prepare_one<T, MM, false, EpiResid>()) != cudaSuccess) return e;
+  return prepare_one<T, MM, true, EpiHead>();
 }
 
 cudaError_t prepare_gemv_kernels() {
@@ -755,7 +1004,7 @@ static cudaError_t part_t(const Dims& D, const Bufs& B, const LayerW& w, int lay
       a.gnorm = w.attn_norm;
       a.x = B.h;
       a.ss_in = 0;
-      return stream_launch<T, MM>(a, EpiQKV<T>{layer}, st);
+      return stream_launch<T, MM, true>(a, EpiQKV<T>{layer}, st);
     case 1:
       return launch_attention(D, B, std::is_same<T, float>::value ? SSD_DTYPE_F32 : SSD_DTYPE_BF16,
                               layer, sel, MM > 1, st);
@@ -765,21 +1014,21 @@ static cudaError_t part_t(const Dims& D, const Bufs& B, const LayerW& w, int lay
       a.gnorm = nullptr;
       a.x = B.attn_out;
       a.ss_in = -1;
-      return stream_launch<T, MM>(a, EpiResid{1}, st);
+      return stream_launch<T, MM, false>(a, EpiResid{1}, st);
     case 3:
       a.g = make_geom(D, 2 * D.F, D.d, elt, kMapGateUp);
       a.W = w.wgu;
       a.gnorm = w.ffn_norm;
       a.x = B.h;
       a.ss_in = 1;
-      return stream_launch<T, MM>(a, EpiGateUp{}, st);
+      return stream_launch<T, MM, true>(a, EpiGateUp{}, st);
     case 4:
       a.g = make_geom(D, D.d, D.F, elt, kMapLinear);
       a.W = w.wdown;
       a.gnorm = nullptr;
       a.x = B.act;
       a.ss_in = -1;
-      return stream_launch<T, MM>(a, EpiResid{0}, st);
+      return stream_launch<T, MM, false>(a, EpiResid{0}, st);
     default:
       return cudaErrorInvalidValue;
   }
@@ -825,7 +1074,7 @@ static cudaError_t head_t(const Dims& D, const Bufs& B, const void* lm, const vo
   a.gnorm = fn;
   a.x = B.h;
   a.ss_in = 0;
-  return stream_launch<T, MM>(a, EpiHead{topk, logits ? 1 : 0}, st);
+  return stream_launch<T, MM, true>(a, EpiHead{topk, logits ? 1 : 0}, st);
 }
 
 cudaError_t launch_head(const Dims& D, const Bufs& B, int dtype, const void* lm_head,
@@ -850,7 +1099,7 @@ static cudaError_t plain_t(const Dims& D, const Bufs& B, const void* W, int rows
   a.gnorm = nullptr;
   a.x = x;
   a.ss_in = -1;
-  return stream_launch<T, MM>(a, EpiPlain{y}, st);
+  return stream_launch<T, MM, false>(a, EpiPlain{y}, st);
 }
 
 cudaError_t launch_gemv_plain(const Dims& D, const Bufs& B, int dtype, const void* W, int rows,
