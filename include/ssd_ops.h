@@ -68,6 +68,26 @@ ssd_status ssd_op_gemv(ssd_ctx* ctx, int32_t which, int32_t layer, int32_t M, co
 ssd_status ssd_op_layer(ssd_ctx* ctx, int32_t kernel, int32_t layer, int32_t M, int32_t pos0,
                         void* stream);
 
+/* Allocation-free form of ssd_op_gemv (the paper has no counterpart: this is
+ * an interface for callers that cannot allocate device memory, e.g. code that
+ * runs while a CUDA graph is being captured, where cudaMalloc is not a
+ * capturable operation, or a host framework that owns the device's memory
+ * pool and allows no other allocations).  Computes y[m][r] = sum_c W[r][c]
+ * x[m][c] for m < M exactly as ssd_op_gemv, without a context: W (device,
+ * rows x cols, dtype, 16-byte aligned rows), x_dev [M][cols] and y_dev
+ * [M][rows] fp32 (device) are the caller's; the kernel's scratch is a fixed
+ * static device array inside libssd.so (about 1.1 MB, held on every device
+ * that uses it until the process exits).
+ * Limits: 1 <= M <= 17 and rows <= 131072 (SSD_ERR_CAPACITY beyond), cols *
+ * element size a multiple of 16 (SSD_ERR_INVALID_ARG otherwise).
+ * The first call on a device looks up the array's device address and sets
+ * kernel attributes; make that first call before any stream capture.  Every
+ * call clears the scratch's tickets on `stream` and shares the one array, so
+ * calls that overlap on the GPU (other streams, other threads) race.  Enqueued
+ * on `stream`; no synchronisation; allocates nothing. */
+ssd_status ssd_gemv_noalloc(const void* W, int32_t dtype, int32_t rows, int32_t cols,
+                            const float* x_dev, int32_t M, float* y_dev, void* stream);
+
 /* Test fixture: fills dst (device, n elements of dtype) with the seeded
  * synthetic weights of tensor `tid` (see synth/synth.h): element i is
  * synth_weight_f32(seed, tid, i, sigma), rounded to bf16 for SSD_DTYPE_BF16.

@@ -28,6 +28,7 @@
 //    (max, argmax, top-k, log-sum-exp, entropy) merged in a fixed tree.
 #include <math.h>
 
+#include <mutex>
 #include <type_traits>
 
 #include "kernels.h"
@@ -1111,6 +1112,82 @@ cudaError_t launch_gemv_plain(const Dims& D, const Bufs& B, int dtype, const voi
                 : plain_t<float, kMaxM>(D, B, W, rows, cols, x, M, y, st);
 }
 
+
+// ----------------------------------------------- allocation-free variant
+//
+// ssd_gemv_noalloc: the plain weight-streaming product for callers that can
+// not allocate device memory.  Its scratch -- the partial sums of row tiles
+// shared by two blocks, their tickets and an error word -- lives in one
+// file-scope device array instead of a caller-provided workspace.
+
+constexpr int kNoAllocBlocks = 256;   // grid cap (one block per SM)
+constexpr int kNoAllocTiles = 4096;   // row tiles of 32: rows <= 131072
+constexpr size_t kNoAllocPart = sizeof(float) * (size_t)kNoAllocBlocks * 2 * kRT * kMaxM;
+constexpr size_t kNoAllocCount = sizeof(uint32_t) * kNoAllocTiles;
+constexpr size_t kNoAllocCtl = (sizeof(Ctl) + 255) / 256 * 256;
+constexpr size_t kNoAllocBytes = kNoAllocPart + kNoAllocCount + kNoAllocCtl;
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
+
+namespace {
+struct NoAllocDevice {
+  bool ready = false;
+  unsigned char* scratch = nullptr;  // device address of g_noalloc_scratch
+  int sms = 0;
+};
+std::mutex g_noalloc_mu;
+NoAllocDevice g_noalloc_dev[64];
+}  // namespace
+
+}  // namespace ssd
+
+extern "C" ssd_status ssd_gemv_noalloc(const void* W, int32_t dtype, int32_t rows, int32_t cols,
+                                       const float* x_dev, int32_t M, float* y_dev,
+                                       void* stream) {
+  using namespace ssd;
+  if (!W || !x_dev || !y_dev || ((uintptr_t)W & 15u) || ((uintptr_t)x_dev & 15u))
+    return SSD_ERR_INVALID_ARG;
+  if (dtype != SSD_DTYPE_F32 && dtype != SSD_DTYPE_BF16) return SSD_ERR_INVALID_ARG;
+  const int elt = dtype == SSD_DTYPE_BF16 ? 2 : 4;
+  if (rows < 1 || cols < 1 || M < 1 || ((size_t)cols * elt) % 16) return SSD_ERR_INVALID_ARG;
+  if (M > kMaxM || (rows + kRT - 1) / kRT > kNoAllocTiles) return SSD_ERR_CAPACITY;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return SSD_ERR_CUDA;
+  NoAllocDevice nd;
+  {
+    // once per device, with that device current: the array's device address
+    // (the symbol's host-side name is not one), kernel attributes, SM count
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    NoAllocDevice& d = g_noalloc_dev[dev];
+    if (!d.ready) {
+      void* p = nullptr;
+      if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return SSD_ERR_CUDA;
+      if (prepare_gemv_kernels() != cudaSuccess) return SSD_ERR_CUDA;
+      int sms = 0;
+      if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return SSD_ERR_CUDA;
+      d.scratch = static_cast<unsigned char*>(p);
+      d.sms = sms < kNoAllocBlocks ? sms : kNoAllocBlocks;
+      d.ready = true;
+    }
+    nd = d;
+  }
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  Bufs B{};
+  B.gpart = reinterpret_cast<float*>(nd.scratch);
+  B.tile_counter = reinterpret_cast<uint32_t*>(nd.scratch + kNoAllocPart);
+  B.ctl = reinterpret_cast<Ctl*>(nd.scratch + kNoAllocPart + kNoAllocCount);
+  Dims D{};
+  D.num_sms = nd.sms;
+  // tickets and the error word start at zero on every call
+  if (cudaMemsetAsync(B.tile_counter, 0, kNoAllocCount + kNoAllocCtl, st) != cudaSuccess)
+    return SSD_ERR_CUDA;
+  return launch_gemv_plain(D, B, dtype, W, rows, cols, x_dev, M, y_dev, st) == cudaSuccess
+             ? SSD_OK
+             : SSD_ERR_CUDA;
+}
+
+namespace ssd {
 // ----------------------------------------------------------------- probe
 __global__ void k_read_probe(const uint4* __restrict__ src, uint64_t n16, uint32_t* sink) {
   uint32_t acc = 0;
