@@ -2,6 +2,7 @@
 // self-speculative decoding engine (sm_103a).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -135,6 +136,7 @@ struct LayerW {
   const void* ffn_norm;
   const void* wgu;
   const void* wdown;
+  const CUtensorMap* tm[4];  // bf16: tensor maps of wqkv, wo, wgu, wdown (host memory)
 };
 
 // Shapes and buffers every kernel may need.
@@ -149,7 +151,8 @@ struct Bufs {
   float* ss;         // [2][kMaxM] sum of squares of h rows: [0] after down/embed, [1] after O
   float* ss_tile;    // [2][2][max blocks][kMaxM] per-block (running, split) partials of ss
   uint32_t* ss_counter;  // [2] block tickets of the residual kernels
-  float* gpart;      // [num_sms][2][32][kMaxM] partial tile sums of blocks sharing a tile
+  float* gpart;      // partial tile sums of blocks sharing a tile: [num_sms][2][32][kMaxM]
+                     // (fp32 kernels) or [num_sms][2][2][kMaxM][128] (bf16 tensor-core kernels)
   uint32_t* tile_counter;      // [max tiles] tickets of shared tiles
   float* xq;         // [kMaxM][qd] rotated queries
   float* attn_part;  // [kMaxM][Hq][nsplit][hd] unnormalised partial outputs

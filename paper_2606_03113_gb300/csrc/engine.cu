@@ -71,7 +71,8 @@ size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
   b.ss = cv.take<float>(sizeof(float) * 2 * kMaxM);
   b.ss_tile = cv.take<float>(sizeof(float) * 2 * 2 * kMaxM * (size_t)kMaxBlocks);
   b.ss_counter = cv.take<uint32_t>(sizeof(uint32_t) * 2);
-  b.gpart = cv.take<float>(sizeof(float) * (size_t)kMaxBlocks * 2 * 32 * kMaxM);
+  b.gpart = cv.take<float>(sizeof(float) * std::max((size_t)kMaxBlocks * 2 * 32 * kMaxM,
+                                                      tile_part_floats(kMaxBlocks)));
   b.tile_counter = cv.take<uint32_t>(sizeof(uint32_t) * (size_t)d.max_tiles);
 
   b.xq = cv.take<float>(sizeof(float) * kMaxM * d.qd);
@@ -123,6 +124,8 @@ struct ssd_ctx {
   const void* lm_head = nullptr;
   const void* final_norm = nullptr;
   std::vector<LayerW> layers;
+  std::vector<CUtensorMap> wmaps;  // bf16: [L][4] layer matrices, then the LM head
+  TileMaps tmaps{};                // bf16: the input buffers
   cudaStream_t stream = nullptr;
   cudaStream_t cap = nullptr;
   std::string err;
@@ -212,15 +215,26 @@ struct Seq {
     if (e_ != cudaSuccess) return e_;           \
   } while (0)
 
-cudaError_t enqueue_layers(ssd_ctx* x, int l_from, int l_to, RowSel sel, bool big,
+const TileMaps* tile_maps(const ssd_ctx* x) {
+  return x->cfg.dtype == SSD_DTYPE_BF16 ? &x->tmaps : nullptr;
+}
+
+const CUtensorMap* lm_map(const ssd_ctx* x) {
+  return x->cfg.dtype == SSD_DTYPE_BF16 ? &x->wmaps[4 * (size_t)x->cfg.n_layers] : nullptr;
+}
+
+// mrows: the most rows the launches will see (1: the single-row kernels).
+cudaError_t enqueue_layers(ssd_ctx* x, int l_from, int l_to, RowSel sel, int mrows,
                            cudaStream_t st) {
   for (int l = l_from; l < l_to; ++l)
-    GK(launch_layer(x->D, x->B, x->cfg.dtype, x->layers[l], l, sel, big, st));
+    GK(launch_layer(x->D, x->B, x->cfg.dtype, x->layers[l], tile_maps(x), l, sel, mrows, st));
   return cudaSuccess;
 }
 
-cudaError_t enqueue_head(ssd_ctx* x, RowSel sel, bool big, int topk, bool logits, cudaStream_t st) {
-  return launch_head(x->D, x->B, x->cfg.dtype, x->lm_head, x->final_norm, topk, logits, sel, big, st);
+cudaError_t enqueue_head(ssd_ctx* x, RowSel sel, int mrows, int topk, bool logits,
+                         cudaStream_t st) {
+  return launch_head(x->D, x->B, x->cfg.dtype, x->lm_head, lm_map(x), tile_maps(x), x->final_norm,
+                     topk, logits, sel, mrows, st);
 }
 
 // Walk segment j: layers (done, c_j], exit head, decision; nested IF for j+1.
@@ -231,8 +245,8 @@ cudaError_t build_walk(ssd_ctx* x, Seq& s, const std::vector<int>& cands, int j,
   if (!last) GK(cudaGraphConditionalHandleCreate(&next, s.g, 0, 0));
   GK(s.begin());
   if (j == 0) GK(launch_embed(x->D, x->B, x->cfg.dtype, x->embed, rows(kRowsWalk), false, 0, x->cap));
-  GK(enqueue_layers(x, done, cands[j], rows(kRowsWalk), false, x->cap));
-  GK(enqueue_head(x, rows(kRowsWalk), false, x->topk, false, x->cap));
+  GK(enqueue_layers(x, done, cands[j], rows(kRowsWalk), 1, x->cap));
+  GK(enqueue_head(x, rows(kRowsWalk), 1, x->topk, false, x->cap));
   GK(launch_decide(x->D, x->B, kDecideWalk, j, last ? 1 : 0, cands[j], next, 0, x->cap));
   GK(s.end());
   if (last) return cudaSuccess;
@@ -267,16 +281,16 @@ cudaError_t build_draft_phase(ssd_ctx* x, cudaGraph_t body) {
     for (int j = 0; j < J; ++j) {
       Seq c{x, cases[j]};
       GK(c.begin());
-      GK(enqueue_layers(x, 0, cands[j], rows(kRowsDraft), false, x->cap));
+      GK(enqueue_layers(x, 0, cands[j], rows(kRowsDraft), 1, x->cap));
       GK(c.end());
     }
     GK(w.begin());
   } else {
     GK(w.begin());
     GK(launch_embed(x->D, x->B, x->cfg.dtype, x->embed, rows(kRowsDraft), false, 0, x->cap));
-    GK(enqueue_layers(x, 0, cands[0], rows(kRowsDraft), false, x->cap));
+    GK(enqueue_layers(x, 0, cands[0], rows(kRowsDraft), 1, x->cap));
   }
-  GK(enqueue_head(x, rows(kRowsDraft), false, x->topk, false, x->cap));
+  GK(enqueue_head(x, rows(kRowsDraft), 1, x->topk, false, x->cap));
   GK(launch_decide(x->D, x->B, kDecideDraft, 0, 0, 0, 0, hw, x->cap));
   return w.end();
 }
@@ -298,8 +312,9 @@ cudaError_t build_round(ssd_ctx* x, cudaGraph_t g, cudaGraphConditionalHandle ge
   }
   GK(s.begin());
   GK(launch_embed(x->D, x->B, x->cfg.dtype, x->embed, rows(kRowsVerify), spec, 0, x->cap));
-  GK(enqueue_layers(x, 0, x->D.L, rows(kRowsVerify), spec, x->cap));
-  GK(enqueue_head(x, rows(kRowsVerify), spec, x->topk, false, x->cap));
+  const int mrows = spec ? std::min(x->kmax + 1, kMaxM) : 1;
+  GK(enqueue_layers(x, 0, x->D.L, rows(kRowsVerify), mrows, x->cap));
+  GK(enqueue_head(x, rows(kRowsVerify), mrows, x->topk, false, x->cap));
   GK(launch_accept(x->D, x->B, gen, x->cap));
   return s.end();
 }
@@ -354,9 +369,9 @@ ssd_status run_prompt(ssd_ctx* x, int n) {
     const int M = std::min(kPrefillChunk, n - c0);
     const RowSel sel = rows_explicit(c0, M, x->B.pre_tok + c0);
     CK(x, launch_embed(x->D, x->B, x->cfg.dtype, x->embed, sel, true, 0, x->stream));
-    CK(x, enqueue_layers(x, 0, x->D.L, sel, true, x->stream));
+    CK(x, enqueue_layers(x, 0, x->D.L, sel, kPrefillChunk, x->stream));
     if (c0 + M > n - T || c0 + M == n) {
-      CK(x, enqueue_head(x, sel, true, x->topk, false, x->stream));
+      CK(x, enqueue_head(x, sel, kPrefillChunk, x->topk, false, x->stream));
       const int first = std::max(c0, n - T) - c0;
       if (first < M) CK(x, launch_trace_push(x->B, first, M - first, x->stream));
     }
@@ -415,10 +430,13 @@ ssd_status ssd_init_model(const ssd_model_cfg* cfg, const ssd_weights* w, void* 
   if (workspace_bytes < need) return fail(nullptr, SSD_ERR_CAPACITY, "workspace too small");
   if (cfg->head_dim % 32 || cfg->ffn_dim % 16)
     return fail(nullptr, SSD_ERR_UNSUPPORTED, "head_dim must be a multiple of 32, ffn_dim of 16");
+  if (cfg->dtype == SSD_DTYPE_BF16 && cfg->head_dim != 128)
+    return fail(nullptr, SSD_ERR_UNSUPPORTED, "bf16 models need head_dim 128");
   int dev = 0, sms = 0;
   cudaError_t e0 = cudaGetDevice(&dev);
   if (e0 == cudaSuccess) e0 = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e0 == cudaSuccess) e0 = prepare_gemv_kernels();
+  if (e0 == cudaSuccess && cfg->dtype == SSD_DTYPE_BF16) e0 = prepare_tile_kernels();
   if (e0 != cudaSuccess) return cuda_fail(nullptr, "ssd_init_model device query", e0);
   if (const char* v = getenv("SSD_NO_PDL")) g_pdl_enabled = !(v[0] == '1');
   ssd_ctx* x = new ssd_ctx();
@@ -431,7 +449,30 @@ ssd_status ssd_init_model(const ssd_model_cfg* cfg, const ssd_weights* w, void* 
   x->layers.resize(cfg->n_layers);
   for (int l = 0; l < cfg->n_layers; ++l)
     x->layers[l] = LayerW{w->attn_norm[l], w->wqkv[l], w->wo[l], w->ffn_norm[l], w->w_gate_up[l],
-                          w->w_down[l]};
+                          w->w_down[l], {nullptr, nullptr, nullptr, nullptr}};
+  if (cfg->dtype == SSD_DTYPE_BF16) {
+    // tensor maps of every weight matrix and of the input buffers
+    const int L = cfg->n_layers, d = cfg->d_model, F = cfg->ffn_dim;
+    const int qkv = (cfg->n_heads + 2 * cfg->n_kv_heads) * cfg->head_dim;
+    const int qd = cfg->n_heads * cfg->head_dim;
+    x->wmaps.resize(4 * (size_t)L + 1);
+    bool ok = true;
+    for (int l = 0; l < L && ok; ++l) {
+      CUtensorMap* m = &x->wmaps[4 * (size_t)l];
+      ok = encode_weight_map(m, w->wqkv[l], qkv, d) && encode_weight_map(m + 1, w->wo[l], d, qd) &&
+           encode_weight_map(m + 2, w->w_gate_up[l], 2 * F, d) &&
+           encode_weight_map(m + 3, w->w_down[l], d, F);
+      for (int k = 0; k < 4; ++k) x->layers[l].tm[k] = m + k;
+    }
+    ok = ok && encode_weight_map(&x->wmaps[4 * (size_t)L], w->lm_head, cfg->vocab, d) &&
+         encode_input_maps(x->tmaps.h, x->B.h, d) &&
+         encode_input_maps(x->tmaps.attn_out, x->B.attn_out, qd) &&
+         encode_input_maps(x->tmaps.act, x->B.act, F);
+    if (!ok) {
+      delete x;
+      return fail(nullptr, SSD_ERR_CUDA, "tensor-map encoding failed");
+    }
+  }
   x->stream = static_cast<cudaStream_t>(cuda_stream);
   cudaError_t e = cudaStreamCreateWithFlags(&x->cap, cudaStreamNonBlocking);
   if (e != cudaSuccess) {
@@ -696,8 +737,8 @@ ssd_status ssd_forward_exit(ssd_ctx* x, const int32_t* ids, int32_t M, int32_t p
   CK(x, cudaMemcpyAsync(x->B.pre_tok, ids, sizeof(int32_t) * M, cudaMemcpyHostToDevice, x->stream));
   const RowSel sel = rows_explicit(pos0, M, x->B.pre_tok);
   CK(x, launch_embed(x->D, x->B, x->cfg.dtype, x->embed, sel, true, 0, x->stream));
-  CK(x, enqueue_layers(x, 0, l_exit, sel, true, x->stream));
-  CK(x, enqueue_head(x, sel, true, topk, logits != nullptr, x->stream));
+  CK(x, enqueue_layers(x, 0, l_exit, sel, M, x->stream));
+  CK(x, enqueue_head(x, sel, M, topk, logits != nullptr, x->stream));
   std::vector<RowStats> st(M);
   CK(x, cudaMemcpyAsync(st.data(), x->B.stats, sizeof(RowStats) * M, cudaMemcpyDeviceToHost,
                         x->stream));
@@ -792,7 +833,15 @@ ssd_status ssd_op_gemv(ssd_ctx* x, int32_t which, int32_t layer, int32_t M, cons
     default: return fail(x, SSD_ERR_INVALID_ARG, "which must be 0..4");
   }
   cudaStream_t st = stream ? static_cast<cudaStream_t>(stream) : x->stream;
-  CK(x, launch_gemv_plain(x->D, x->B, c.dtype, W, rows, cols, x_dev, M, y_dev, st));
+  if (c.dtype == SSD_DTYPE_BF16) {
+    const CUtensorMap& wm = which == 4 ? x->wmaps[4 * (size_t)c.n_layers]
+                                       : x->wmaps[4 * (size_t)layer + which];
+    if (((uintptr_t)x_dev & 15u) || ((size_t)cols * 4) % 16)
+      return fail(x, SSD_ERR_INVALID_ARG, "x_dev must be 16-byte aligned");
+    CK(x, launch_tile_plain(x->D, x->B, wm, rows, cols, x_dev, M, y_dev, st));
+  } else {
+    CK(x, launch_gemv_plain(x->D, x->B, c.dtype, W, rows, cols, x_dev, M, y_dev, st));
+  }
   return SSD_OK;
 }
 
@@ -805,12 +854,11 @@ ssd_status ssd_op_layer(ssd_ctx* x, int32_t kernel, int32_t layer, int32_t M, in
     return fail(x, SSD_ERR_INVALID_ARG, "kernel must be 0..5 and layer in range");
   cudaStream_t st = stream ? static_cast<cudaStream_t>(stream) : x->stream;
   const RowSel sel = rows_explicit(pos0, M, x->B.pre_tok);
-  const bool big = M > 1;
   if (kernel == 5)
-    CK(x, enqueue_head(x, sel, big, x->topk, false, st));
+    CK(x, enqueue_head(x, sel, M, x->topk, false, st));
   else
-    CK(x, launch_layer_part(x->D, x->B, x->cfg.dtype, x->layers[kernel == 5 ? 0 : layer], layer,
-                            kernel, sel, big, st));
+    CK(x, launch_layer_part(x->D, x->B, x->cfg.dtype, x->layers[layer], tile_maps(x), layer,
+                            kernel, sel, M, st));
   return SSD_OK;
 }
 

@@ -31,6 +31,7 @@
 #include <mutex>
 #include <type_traits>
 
+#include "headpart.cuh"
 #include "kernels.h"
 #include "pipe.cuh"
 
@@ -148,126 +149,6 @@ struct Shared {
 // the dot products v0, v1.  Kernels with a running result (residual norm sums,
 // exit-head statistics) keep per-lane state; finish() combines it once per
 // block and the last block reduces the blocks in a fixed order.
-
-__device__ __forceinline__ bool better(float v1, int i1, float v2, int i2) {
-  return v1 > v2 || (v1 == v2 && i1 < i2);
-}
-
-__device__ inline void part_empty(HeadPart& p) {
-  p.mx = -INFINITY;
-  p.S = 0.f;
-  p.T = 0.f;
-#pragma unroll
-  for (int q = 0; q < kTopK; ++q) {
-    p.tv[q] = -INFINITY;
-    p.ti[q] = 0x7fffffff;
-  }
-}
-
-// Inserts (v, idx) into the descending top-k list with compare-swaps at fixed
-// positions (no runtime indexing, so the list stays in registers).
-__device__ __forceinline__ void topk_insert(float (&tv)[kTopK], int (&ti)[kTopK], float v, int idx) {
-#pragma unroll
-  for (int q = 0; q < kTopK; ++q) {
-    const bool b = better(v, idx, tv[q], ti[q]);
-    const float tvq = tv[q];
-    const int tiq = ti[q];
-    tv[q] = b ? v : tvq;
-    ti[q] = b ? idx : tiq;
-    v = b ? tvq : v;
-    idx = b ? tiq : idx;
-  }
-}
-
-__device__ __forceinline__ void cswap(float (&tv)[kTopK], int (&ti)[kTopK], int i, int j) {
-  const bool keep = better(tv[i], ti[i], tv[j], ti[j]);
-  const float a = tv[i], b = tv[j];
-  const int ia = ti[i], ib = ti[j];
-  tv[i] = keep ? a : b;
-  ti[i] = keep ? ia : ib;
-  tv[j] = keep ? b : a;
-  ti[j] = keep ? ib : ia;
-}
-
-// a <- merge(a, b); symmetric in a and b (max, commutative sums, a total
-// order on (value, index)), so both lanes of a shuffle exchange compute the
-// same result.  Top-k: bitonic merge of the two sorted lists (elementwise
-// best of a[i] and b[k-1-i], then a sorting network of 12 compare-swaps).
-__device__ inline void part_merge(HeadPart& a, const HeadPart& b) {
-  static_assert(kTopK == 8, "bitonic network written for 8");
-  if (b.S > 0.f) {
-    if (a.S > 0.f) {
-      const float mx = fmaxf(a.mx, b.mx);
-      const float ea = expf(a.mx - mx), eb = expf(b.mx - mx);
-      const float S = a.S * ea + b.S * eb;
-      const float Tt = ea * (a.T + (a.mx - mx) * a.S) + eb * (b.T + (b.mx - mx) * b.S);
-      a.mx = mx;
-      a.S = S;
-      a.T = Tt;
-    } else {
-      a.mx = b.mx;
-      a.S = b.S;
-      a.T = b.T;
-    }
-  }
-#pragma unroll
-  for (int i = 0; i < kTopK; ++i) {
-    const bool keep = better(a.tv[i], a.ti[i], b.tv[kTopK - 1 - i], b.ti[kTopK - 1 - i]);
-    a.tv[i] = keep ? a.tv[i] : b.tv[kTopK - 1 - i];
-    a.ti[i] = keep ? a.ti[i] : b.ti[kTopK - 1 - i];
-  }
-#pragma unroll
-  for (int i = 0; i < 4; ++i) cswap(a.tv, a.ti, i, i + 4);
-  cswap(a.tv, a.ti, 0, 2);
-  cswap(a.tv, a.ti, 1, 3);
-  cswap(a.tv, a.ti, 4, 6);
-  cswap(a.tv, a.ti, 5, 7);
-#pragma unroll
-  for (int i = 0; i < 8; i += 2) cswap(a.tv, a.ti, i, i + 1);
-}
-
-// Adds one logit z of vocabulary row idx.
-__device__ inline void part_add(HeadPart& p, float z, int idx) {
-  if (!(z > -INFINITY)) return;
-  if (p.S > 0.f) {
-    const float mx = fmaxf(p.mx, z);
-    const float e_old = expf(p.mx - mx), e_new = expf(z - mx);
-    p.T = e_old * (p.T + (p.mx - mx) * p.S) + e_new * (z - mx);
-    p.S = p.S * e_old + e_new;
-    p.mx = mx;
-  } else {
-    p.mx = z;
-    p.S = 1.f;
-    p.T = 0.f;
-  }
-  topk_insert(p.tv, p.ti, z, idx);
-}
-
-__device__ inline HeadPart part_shfl(const HeadPart& p, int off) {
-  HeadPart q;
-  q.mx = __shfl_xor_sync(0xffffffffu, p.mx, off);
-  q.S = __shfl_xor_sync(0xffffffffu, p.S, off);
-  q.T = __shfl_xor_sync(0xffffffffu, p.T, off);
-#pragma unroll
-  for (int t = 0; t < kTopK; ++t) {
-    q.tv[t] = __shfl_xor_sync(0xffffffffu, p.tv[t], off);
-    q.ti[t] = __shfl_xor_sync(0xffffffffu, p.ti[t], off);
-  }
-  return q;
-}
-
-__device__ inline HeadPart part_load_cg(const HeadPart* src) {
-  HeadPart q;
-  q.mx = __ldcg(&src->mx);
-  q.S = __ldcg(&src->S);
-  q.T = __ldcg(&src->T);
-#pragma unroll
-  for (int t = 0; t < kTopK; ++t) {
-    q.tv[t] = __ldcg(&src->tv[t]);
-    q.ti[t] = __ldcg(&src->ti[t]);
-  }
-  return q;
-}
 
 struct NoState {};
 
@@ -516,22 +397,7 @@ struct EpiHead {
           part_empty(f);
         for (int off = 4; off > 0; off >>= 1) part_merge(f, part_shfl(f, off));
         if (lane == 0) {
-          RowStats& o = a.B.stats[m];
-          const float logS = logf(f.S);
-          o.argmax = f.ti[0];
-          o.zmax = f.mx;
-          o.lse = f.mx + logS;
-          o.entropy = logS - f.T / f.S;
-          float tsum = 0.f;
-#pragma unroll
-          for (int q = 0; q < kTopK; ++q) {
-            o.top_idx[q] = f.ti[q];
-            o.top_logit[q] = f.tv[q];
-            if (q < topk) tsum += f.tv[q];
-          }
-          o.conf_k = o.lse - tsum / (float)topk;
-          o.pmax = 1.0f / f.S;
-          o.margin = f.tv[0] - f.tv[1];
+          write_row_stats(a.B.stats[m], f, topk);
         }
       }
       named_sync(1, kCThreads);
@@ -982,8 +848,10 @@ cudaError_t prepare_gemv_kernels() {
   cudaError_t e;
   if ((e = prepare_t<float, 1>()) != cudaSuccess) return e;
   if ((e = prepare_t<float, kMaxM>()) != cudaSuccess) return e;
-  if ((e = prepare_t<__nv_bfloat16, 1>()) != cudaSuccess) return e;
-  return prepare_t<__nv_bfloat16, kMaxM>();
+  // bf16 models run on the tensor-core kernels (tile.cu); the plain bf16
+  // product stays here for the allocation-free entry point
+  if ((e = prepare_one<__nv_bfloat16, 1, false, EpiPlain>()) != cudaSuccess) return e;
+  return prepare_one<__nv_bfloat16, kMaxM, false, EpiPlain>();
 }
 
 // Attention launchers live in attention.cu.
@@ -1035,32 +903,26 @@ static cudaError_t part_t(const Dims& D, const Bufs& B, const LayerW& w, int lay
   }
 }
 
-template <typename T, int MM>
-static cudaError_t layer_t(const Dims& D, const Bufs& B, const LayerW& w, int layer, RowSel sel,
-                           cudaStream_t st) {
-  for (int part = 0; part < kLayerKernels - 1; ++part) {
-    cudaError_t e = part_t<T, MM>(D, B, w, layer, part, sel, st);
-    if (e != cudaSuccess) return e;
+cudaError_t launch_layer_part(const Dims& D, const Bufs& B, int dtype, const LayerW& w,
+                              const TileMaps* tm, int layer, int part, RowSel sel, int mrows,
+                              cudaStream_t st) {
+  const bool big = mrows > 1;
+  if (dtype == SSD_DTYPE_BF16) {
+    if (part == 1) return launch_attention(D, B, dtype, layer, sel, big, st);
+    if (!tm) return cudaErrorInvalidValue;
+    return launch_tile_part(D, B, *tm, w, layer, part, sel, mrows, st);
   }
-  return cudaSuccess;
-}
-
-cudaError_t launch_layer_part(const Dims& D, const Bufs& B, int dtype, const LayerW& w, int layer,
-                              int part, RowSel sel, bool big, cudaStream_t st) {
-  if (dtype == SSD_DTYPE_BF16)
-    return big ? part_t<__nv_bfloat16, kMaxM>(D, B, w, layer, part, sel, st)
-               : part_t<__nv_bfloat16, 1>(D, B, w, layer, part, sel, st);
   return big ? part_t<float, kMaxM>(D, B, w, layer, part, sel, st)
              : part_t<float, 1>(D, B, w, layer, part, sel, st);
 }
 
-cudaError_t launch_layer(const Dims& D, const Bufs& B, int dtype, const LayerW& w, int layer,
-                         RowSel sel, bool big, cudaStream_t st) {
-  if (dtype == SSD_DTYPE_BF16)
-    return big ? layer_t<__nv_bfloat16, kMaxM>(D, B, w, layer, sel, st)
-               : layer_t<__nv_bfloat16, 1>(D, B, w, layer, sel, st);
-  return big ? layer_t<float, kMaxM>(D, B, w, layer, sel, st)
-             : layer_t<float, 1>(D, B, w, layer, sel, st);
+cudaError_t launch_layer(const Dims& D, const Bufs& B, int dtype, const LayerW& w,
+                         const TileMaps* tm, int layer, RowSel sel, int mrows, cudaStream_t st) {
+  for (int part = 0; part < kLayerKernels - 1; ++part) {
+    cudaError_t e = launch_layer_part(D, B, dtype, w, tm, layer, part, sel, mrows, st);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 template <typename T, int MM>
@@ -1079,13 +941,14 @@ static cudaError_t head_t(const Dims& D, const Bufs& B, const void* lm, const vo
 }
 
 cudaError_t launch_head(const Dims& D, const Bufs& B, int dtype, const void* lm_head,
-                        const void* final_norm, int topk, bool write_logits, RowSel sel, bool big,
-                        cudaStream_t st) {
-  if (dtype == SSD_DTYPE_BF16)
-    return big ? head_t<__nv_bfloat16, kMaxM>(D, B, lm_head, final_norm, topk, write_logits, sel, st)
-               : head_t<__nv_bfloat16, 1>(D, B, lm_head, final_norm, topk, write_logits, sel, st);
-  return big ? head_t<float, kMaxM>(D, B, lm_head, final_norm, topk, write_logits, sel, st)
-             : head_t<float, 1>(D, B, lm_head, final_norm, topk, write_logits, sel, st);
+                        const CUtensorMap* lm_map, const TileMaps* tm, const void* final_norm,
+                        int topk, bool write_logits, RowSel sel, int mrows, cudaStream_t st) {
+  if (dtype == SSD_DTYPE_BF16) {
+    if (!tm || !lm_map) return cudaErrorInvalidValue;
+    return launch_tile_head(D, B, *tm, *lm_map, final_norm, topk, write_logits, sel, mrows, st);
+  }
+  return mrows > 1 ? head_t<float, kMaxM>(D, B, lm_head, final_norm, topk, write_logits, sel, st)
+                   : head_t<float, 1>(D, B, lm_head, final_norm, topk, write_logits, sel, st);
 }
 
 template <typename T, int MM>

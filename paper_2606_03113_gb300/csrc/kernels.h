@@ -19,18 +19,43 @@ struct HeadPart {
 constexpr int kMaxBlocks = 512;
 inline int head_tiles(int V) { return (V + 15) / 16; }
 
-// big = true selects the kernels instantiated for up to kMaxM rows; false
-// the single-row ones.
+// Tensor maps of the engine's fp32 input buffers ([kMaxM][K] each), read by
+// the bf16 tensor-core kernels one 64-column slice per unit.
+struct TileMaps {
+  CUtensorMap h[3], attn_out[3], act[3];  // boxes of 8, 16, 24 rows
+};
+
+// Encodes the tensor map of a bf16 weight matrix [rows][cols] (64 x 64 boxes,
+// 128-byte swizzle) or of an fp32 input [rows][cols] (64 x kMaxM boxes).
+bool encode_weight_map(CUtensorMap* m, const void* W, int rows, int cols);
+bool encode_input_map(CUtensorMap* m, const float* x, int cols, int rows, int box_rows);
+bool encode_input_maps(CUtensorMap (&m)[3], const float* x, int cols);
+cudaError_t prepare_tile_kernels();
+// Floats of the tensor-core kernels' split-tile partials for `num_sms` blocks.
+size_t tile_part_floats(int num_sms);
+cudaError_t launch_tile_part(const Dims& D, const Bufs& B, const TileMaps& tm, const LayerW& w,
+                             int layer, int part, RowSel sel, int mrows, cudaStream_t st);
+cudaError_t launch_tile_head(const Dims& D, const Bufs& B, const TileMaps& tm,
+                             const CUtensorMap& lm, const void* final_norm, int topk,
+                             bool write_logits, RowSel sel, int mrows, cudaStream_t st);
+cudaError_t launch_tile_plain(const Dims& D, const Bufs& B, const CUtensorMap& wm, int rows,
+                              int cols, const float* x, int M, float* y, cudaStream_t st);
+
+// mrows is the largest number of rows a launch may see: 1 selects the
+// single-row kernels, more the multi-row ones (bf16: the tensor-core instance
+// with 8, 16 or 24 token rows, the smallest that holds mrows).  big
+// (embedding, attention) is mrows > 1.
 cudaError_t launch_embed(const Dims& D, const Bufs& B, int dtype, const void* embed, RowSel sel,
                          bool big, cudaGraphConditionalHandle set_lstar_switch, cudaStream_t st);
-cudaError_t launch_layer(const Dims& D, const Bufs& B, int dtype, const LayerW& w, int layer,
-                         RowSel sel, bool big, cudaStream_t st);
+cudaError_t launch_layer(const Dims& D, const Bufs& B, int dtype, const LayerW& w,
+                         const TileMaps* tm, int layer, RowSel sel, int mrows, cudaStream_t st);
 // One kernel of a layer (0 qkv, 1 attention + combine, 2 o, 3 gate/up, 4 down).
-cudaError_t launch_layer_part(const Dims& D, const Bufs& B, int dtype, const LayerW& w, int layer,
-                              int part, RowSel sel, bool big, cudaStream_t st);
+cudaError_t launch_layer_part(const Dims& D, const Bufs& B, int dtype, const LayerW& w,
+                              const TileMaps* tm, int layer, int part, RowSel sel, int mrows,
+                              cudaStream_t st);
 cudaError_t launch_head(const Dims& D, const Bufs& B, int dtype, const void* lm_head,
-                        const void* final_norm, int topk, bool write_logits, RowSel sel, bool big,
-                        cudaStream_t st);
+                        const CUtensorMap* lm_map, const TileMaps* tm, const void* final_norm,
+                        int topk, bool write_logits, RowSel sel, int mrows, cudaStream_t st);
 cudaError_t launch_round_begin(const Dims& D, const Bufs& B, cudaGraphConditionalHandle draft_if,
                                cudaStream_t st);
 cudaError_t launch_decide(const Dims& D, const Bufs& B, int mode, int cand_idx, int is_last,
