@@ -142,6 +142,7 @@ struct LayerW {
 // Shapes and buffers every kernel may need.
 struct Dims {
   int32_t L, d, Hq, Hkv, hd, F, V, max_seq, qd, kvd, nsplit, num_sms, ss_tiles, max_tiles;
+  int32_t ss_nt;  // 256-row tiles of a residual row (tensor-core kernels' sum-of-squares parts)
   float eps;
 };
 
@@ -151,6 +152,9 @@ struct Bufs {
   float* ss;         // [2][kMaxM] sum of squares of h rows: [0] after down/embed, [1] after O
   float* ss_tile;    // [2][2][max blocks][kMaxM] per-block (running, split) partials of ss
   uint32_t* ss_counter;  // [2] block tickets of the residual kernels
+  float* ss_part;    // [2][ss_nt][kMaxM] sum of squares of h rows per 256-row tile (bf16
+                     // kernels): written by the tile that finishes those rows, summed in
+                     // tile order by the RMSNorm that reads them
   float* gpart;      // partial tile sums of blocks sharing a tile: [num_sms][2][32][kMaxM]
                      // (fp32 kernels) or [num_sms][2][2][kMaxM][128] (bf16 tensor-core kernels)
   uint32_t* tile_counter;      // [max tiles] tickets of shared tiles

@@ -59,6 +59,18 @@ __global__ void k_embed(Dims D, Bufs B, const T* __restrict__ emb, RowSel sel,
   }
   const T* row = emb + (size_t)tok * D.d;
   float* hr = B.h + (size_t)m * D.d;
+  // sums of squares per 256-element part (one warp per part), as the
+  // tensor-core kernels' residual epilogues write them
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int c = warp; c < D.ss_nt; c += (int)(blockDim.x >> 5)) {
+    float sp = 0.f;
+    for (int i = c * 256 + lane; i < min(D.d, c * 256 + 256); i += 32) {
+      const float v = Elem<T>::to_f(row[i]);
+      sp = fmaf(v, v, sp);
+    }
+    sp = warp_sum(sp);
+    if (lane == 0) B.ss_part[(size_t)c * kMaxM + m] = sp;
+  }
   float ss = 0.f;
   for (int i = threadIdx.x; i < D.d; i += blockDim.x) {
     const float v = Elem<T>::to_f(row[i]);

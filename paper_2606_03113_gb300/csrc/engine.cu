@@ -60,6 +60,7 @@ size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
   d.eps = c.rms_eps;
   d.num_sms = kMaxBlocks;  // set to the device's SM count at init
   d.ss_tiles = (c.d_model + 15) / 16;
+  d.ss_nt = (c.d_model + 255) / 256;
   d.max_tiles = std::max(
       std::max(head_tiles(c.vocab), c.ffn_dim / 16 + 1),
       std::max((c.n_heads + 2 * c.n_kv_heads) * c.head_dim / 16 + 2, c.d_model / 16 + 1));
@@ -71,6 +72,7 @@ size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
   b.ss = cv.take<float>(sizeof(float) * 2 * kMaxM);
   b.ss_tile = cv.take<float>(sizeof(float) * 2 * 2 * kMaxM * (size_t)kMaxBlocks);
   b.ss_counter = cv.take<uint32_t>(sizeof(uint32_t) * 2);
+  b.ss_part = cv.take<float>(sizeof(float) * 2 * (size_t)d.ss_nt * kMaxM);
   b.gpart = cv.take<float>(sizeof(float) * std::max((size_t)kMaxBlocks * 2 * 32 * kMaxM,
                                                       tile_part_floats(kMaxBlocks)));
   b.tile_counter = cv.take<uint32_t>(sizeof(uint32_t) * (size_t)d.max_tiles);
@@ -494,6 +496,8 @@ ssd_status ssd_init_model(const ssd_model_cfg* cfg, const ssd_weights* w, void* 
   if (e == cudaSuccess) e = cudaMemsetAsync(x->B.ctl, 0, sizeof(Ctl), x->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(x->B.head_counter, 0, sizeof(uint32_t), x->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(x->B.ss, 0, sizeof(float) * 2 * kMaxM, x->stream);
+  if (e == cudaSuccess)
+    e = cudaMemsetAsync(x->B.ss_part, 0, sizeof(float) * 2 * (size_t)x->D.ss_nt * kMaxM, x->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(x->B.ss_counter, 0, sizeof(uint32_t) * 2, x->stream);
   if (e == cudaSuccess)
     e = cudaMemsetAsync(x->B.tile_counter, 0, sizeof(uint32_t) * (size_t)x->D.max_tiles, x->stream);

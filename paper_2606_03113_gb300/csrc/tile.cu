@@ -96,7 +96,7 @@ struct TGeom {
   int N, K;          // rows, columns
   int nks;           // units per tile (64-column chunks)
   int ntiles;
-  long long T;       // units
+  int T;            // units (T * kMaxBlocks < 2^31, checked by the launcher)
   int P;             // blocks
   int map;
 };
@@ -114,12 +114,14 @@ struct TArgs {
   float* y;                    // plain product output [M][N]
 };
 
-__host__ __device__ inline long long t_start(const TGeom& g, int b) {
-  return g.T * (long long)b / g.P;
+// First unit of block b.  32-bit arithmetic: the split-tile fix-ups evaluate
+// this for every contributor, and 64-bit division would dominate them.
+__host__ __device__ inline int t_start(const TGeom& g, int b) {
+  return (int)((unsigned)g.T * (unsigned)b / (unsigned)g.P);
 }
 
-__device__ inline int t_block_of(const TGeom& g, long long s) {
-  int b = (int)(s * g.P / g.T);
+__device__ inline int t_block_of(const TGeom& g, int s) {
+  int b = (int)((unsigned)s * (unsigned)g.P / (unsigned)g.T);
   if (b >= g.P) b = g.P - 1;
   while (b + 1 < g.P && t_start(g, b + 1) <= s) ++b;
   while (b > 0 && t_start(g, b) > s) --b;
@@ -129,9 +131,9 @@ __device__ inline int t_block_of(const TGeom& g, long long s) {
 // Block b owns the split slot of the tile it starts and shares with the next
 // block(s), if its last tile is such a tile.
 __device__ inline bool t_has_split_slot(const TGeom& g, int b) {
-  const long long sb = t_start(g, b), se = t_start(g, b + 1);
+  const int sb = t_start(g, b), se = t_start(g, b + 1);
   if (se <= sb) return false;
-  const long long t = (se - 1) / g.nks;
+  const int t = (se - 1) / g.nks;
   if ((t + 1) * g.nks <= se) return false;
   return t * g.nks >= sb;
 }
@@ -302,7 +304,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
 
   const TGeom& g = a.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
-  const long long u_begin = t_start(g, blockIdx.x), u_end = t_start(g, blockIdx.x + 1);
+  const int u_begin = t_start(g, blockIdx.x), u_end = t_start(g, blockIdx.x + 1);
   const int n = (int)(u_end - u_begin);
 
   if (tid == 0) {
@@ -336,8 +338,8 @@ __global__ void __launch_bounds__(kTThreads, 1)
       auto issue_w = [&](int i) -> bool {
         const int slot = i % NS;
         if (!mbar_wait(&empty[slot], ((uint32_t)(i / NS) & 1u) ^ 1u)) return false;
-        const long long u = u_begin + i;
-        const int tile = (int)(u / g.nks), kc = (int)(u - (long long)tile * g.nks);
+        const int u = u_begin + i;
+        const int tile = u / g.nks, kc = u - tile * g.nks;
         mbar_arrive_expect_tx(&full[slot], (uint32_t)kWBytes);
         unsigned char* dst = smem + S::ring + (size_t)slot * kWBytes;
 #pragma unroll
@@ -377,7 +379,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
       bool ok = true;
       int tc = -1;
       for (int i = 0; i < n && ok; ++i) {
-        const long long u = u_begin + i;
+        const int u = u_begin + i;
         const int slot = i % NS;
         const uint32_t ph = (uint32_t)(i / NS) & 1u;
         const bool first = (i == 0) || (u % g.nks == 0);
@@ -413,9 +415,16 @@ __global__ void __launch_bounds__(kTThreads, 1)
     resolve_rows(a.B.ctl, a.sel, pos0, M);
     if (M > TP) M = TP;  // the launcher picks TP >= M
     if (tid < 32) {
+      // RMSNorm scale of row tid: the input's sum of squares is kept as parts
+      // of 256 elements, added here in part order
       float r = 1.f;
-      if (a.ss_in >= 0 && tid < M)
-        r = 1.0f / sqrtf(a.B.ss[a.ss_in * kMaxM + tid] / (float)g.K + a.D.eps);
+      if (a.ss_in >= 0 && tid < M) {
+        const float* sp = a.B.ss_part + (size_t)a.ss_in * a.D.ss_nt * kMaxM + tid;
+        float sum = 0.f;
+#pragma unroll 8
+        for (int c = 0; c < a.D.ss_nt; ++c) sum += __ldcg(&sp[(size_t)c * kMaxM]);
+        r = 1.0f / sqrtf(sum / (float)g.K + a.D.eps);
+      }
       srs[tid] = r;
     }
     {
@@ -431,11 +440,26 @@ __global__ void __launch_bounds__(kTThreads, 1)
     float rs_t[LTN];
 #pragma unroll
     for (int lt = 0; lt < LTN; ++lt) rs_t[lt] = srs[2 * lt + grp];
-    float ss_run[LTN];
-#pragma unroll
-    for (int lt = 0; lt < LTN; ++lt) ss_run[lt] = 0.f;
     bool ok = true;
     const int first_tile = (int)(u_begin / g.nks);
+
+    // Residual kernels: sum of squares of the tile's 256 updated rows per
+    // token (fixed order: lanes, then the four row quarters), one part of the
+    // next RMSNorm's input
+    auto tile_ss = [&](const float (&ssv)[LTN], int tile) {
+#pragma unroll
+      for (int lt = 0; lt < LTR; ++lt) {
+        const float sw = warp_sum(ssv[lt]);
+        if (lane == 0) red[warp * kLT + lt] = sw;
+      }
+      named_sync(1, kWThreads);
+      if (tid < M) {
+        float sum = 0.f;
+        for (int qq = 0; qq < 4; ++qq) sum += red[((tid & 1) * 4 + qq) * kLT + (tid >> 1)];
+        a.B.ss_part[((size_t)a.which * a.D.ss_nt + tile) * kMaxM + tid] = sum;
+      }
+      named_sync(1, kWThreads);
+    };
 
     // per-tile epilogue: TMEM -> registers (high + low parts) -> fused epilogue
     auto epilogue = [&](int tile, int tc) {
@@ -468,8 +492,11 @@ __global__ void __launch_bounds__(kTThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&accempty[buf]);
-      const long long t0 = (long long)tile * g.nks, t1 = t0 + g.nks;
+      const int t0 = tile * g.nks, t1 = t0 + g.nks;
       if (t0 >= u_begin && t1 <= u_end) {
+        float ssv[LTN];
+#pragma unroll
+        for (int lt = 0; lt < LTN; ++lt) ssv[lt] = 0.f;
 #pragma unroll
         for (int lt = 0; lt < LTN; ++lt) {
           const int t = 2 * lt + grp;
@@ -479,8 +506,9 @@ __global__ void __launch_bounds__(kTThreads, 1)
           if constexpr (KIND == kKHead)
             t_head_token(a, tile, srow, t, rs_t[lt], v0, v1, &run[warp * kLT + lt], lane);
           else
-            t_pair<KIND>(a, tile, srow, t, pos0, rs_t[lt], v0, v1, ss_run[lt]);
+            t_pair<KIND>(a, tile, srow, t, pos0, rs_t[lt], v0, v1, ssv[lt]);
         }
+        if constexpr (KIND == kKResid) tile_ss(ssv, tile);
         return;
       }
       // shared with neighbouring blocks: publish this block's partial sums
@@ -513,38 +541,85 @@ __global__ void __launch_bounds__(kTThreads, 1)
           for (int lt = 0; lt < kLT; ++lt) part_empty(spl[warp * kLT + lt]);
         __syncwarp();
       }
+      // Partial sums of the contributors, added in block order (independent of
+      // who finishes last).  The loads of several contributors (and all
+      // tokens) are issued before any is used, so the fix-up costs a few L2
+      // round trips rather than one per contributor and token.  Unused slots
+      // read block 0's partials (valid memory) and add zero.
+      constexpr int GB = LTN <= 4 ? 4 : (LTN <= 8 ? 2 : 1);
+      float u0[LTN], u1[LTN];
+#pragma unroll
+      for (int lt = 0; lt < LTN; ++lt) u0[lt] = u1[lt] = 0.f;
+      if (M == 1) {
+        // one token (drafting, autoregressive steps): eight contributors per round
+        for (int b = grp == 0 ? b0 : b1 + 1; b <= b1; b += 8) {
+          float c0[8], c1[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int bb = b + j;
+            bool use = false;
+            int sl = 0;
+            if (bb <= b1) {
+              const int sb = t_start(g, bb);
+              use = sb != t_start(g, bb + 1);
+              sl = tile == (int)(sb / g.nks) ? 0 : 1;
+            }
+            const float* p = a.B.gpart + ((size_t)(use ? bb : 0) * 2 + sl) * 2 * kMaxM * 128;
+            const float x0 = __ldcg(&p[srow]);
+            const float x1 = __ldcg(&p[(size_t)kMaxM * 128 + srow]);
+            c0[j] = use ? x0 : 0.f;
+            c1[j] = use ? x1 : 0.f;
+          }
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            u0[0] += c0[j];
+            u1[0] += c1[j];
+          }
+        }
+      } else for (int b = b0; b <= b1; b += GB) {
+        float c0[GB][LTN], c1[GB][LTN];
+#pragma unroll
+        for (int j = 0; j < GB; ++j) {
+          const int bb = b + j;
+          bool use = false;
+          int sl = 0;
+          if (bb <= b1) {
+            const int sb = t_start(g, bb);
+            use = sb != t_start(g, bb + 1);
+            sl = tile == (int)(sb / g.nks) ? 0 : 1;
+          }
+          const float* p = a.B.gpart + ((size_t)(use ? bb : 0) * 2 + sl) * 2 * kMaxM * 128;
+#pragma unroll
+          for (int lt = 0; lt < LTN; ++lt) {
+            const int t = 2 * lt + grp;
+            const int tt = t < M ? t : 0;
+            const float x0 = __ldcg(&p[(size_t)tt * 128 + srow]);
+            const float x1 = __ldcg(&p[(size_t)(kMaxM + tt) * 128 + srow]);
+            c0[j][lt] = use ? x0 : 0.f;
+            c1[j][lt] = use ? x1 : 0.f;
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < GB; ++j)
+#pragma unroll
+          for (int lt = 0; lt < LTN; ++lt) {
+            u0[lt] += c0[j][lt];
+            u1[lt] += c1[j][lt];
+          }
+      }
 #pragma unroll
       for (int lt = 0; lt < LTN; ++lt) {
         const int t = 2 * lt + grp;
         if (t >= M) break;
-        float u0 = 0.f, u1 = 0.f;
-        for (int b = b0; b <= b1; ++b) {  // block order: independent of who finishes
-          const long long sb = t_start(g, b);
-          if (sb == t_start(g, b + 1)) continue;
-          const int sl = tile == (int)(sb / g.nks) ? 0 : 1;
-          const float* p = a.B.gpart + ((size_t)b * 2 + sl) * 2 * kMaxM * 128;
-          u0 += __ldcg(&p[(size_t)t * 128 + srow]);
-          u1 += __ldcg(&p[(size_t)(kMaxM + t) * 128 + srow]);
-        }
         if constexpr (KIND == kKHead)
-          t_head_token(a, tile, srow, t, rs_t[lt], u0, u1, &spl[warp * kLT + lt], lane);
+          t_head_token(a, tile, srow, t, rs_t[lt], u0[lt], u1[lt], &spl[warp * kLT + lt], lane);
         else
-          t_pair<KIND>(a, tile, srow, t, pos0, rs_t[lt], u0, u1, ss_sp[lt]);
+          t_pair<KIND>(a, tile, srow, t, pos0, rs_t[lt], u0[lt], u1[lt], ss_sp[lt]);
       }
-      // the split tile's statistics go to the split slot of its first block
+      // the split tile's statistics: residual sums of squares as the tile's
+      // part; exit-head statistics to the split slot of its first block
       if constexpr (KIND == kKResid) {
-#pragma unroll
-        for (int lt = 0; lt < LTR; ++lt) {
-          const float s = warp_sum(ss_sp[lt]);
-          if (lane == 0) red[warp * kLT + lt] = s;
-        }
-        named_sync(1, kWThreads);
-        if (tid < M) {
-          float s = 0.f;
-          for (int qq = 0; qq < 4; ++qq) s += red[((tid & 1) * 4 + qq) * kLT + (tid >> 1)];
-          a.B.ss_tile[((size_t)a.which * 2 * kMaxBlocksDev + kMaxBlocksDev + b0) * kMaxM + tid] = s;
-        }
-        named_sync(1, kWThreads);
+        tile_ss(ss_sp, tile);
       } else if constexpr (KIND == kKHead) {
         named_sync(1, kWThreads);
         if (tid < M) {
@@ -560,9 +635,9 @@ __global__ void __launch_bounds__(kTThreads, 1)
     int tc = -1;
     int prev_tile = -1;
     for (int i = 0; i < n; ++i) {
-      const long long u = u_begin + i;
+      const int u = u_begin + i;
       const int slot = i % NS;
-      const int tile = (int)(u / g.nks), kc = (int)(u - (long long)tile * g.nks);
+      const int tile = u / g.nks, kc = u - tile * g.nks;
       if (i == 0 || kc == 0) ++tc;
       // operand tile of unit i, built while its weights are still in flight:
       // the slot's previous use was released before its copies were issued,
@@ -615,45 +690,8 @@ __global__ void __launch_bounds__(kTThreads, 1)
     }
     if (n > 0) epilogue(prev_tile, tc);
 
-    // ---- per-block statistics, and the last block's fixed-order merge
-    if constexpr (KIND == kKResid) {
-      float* sl = a.B.ss_tile + (size_t)a.which * 2 * kMaxBlocksDev * kMaxM;
-#pragma unroll
-      for (int lt = 0; lt < LTR; ++lt) {
-        const float s = warp_sum(ss_run[lt]);
-        if (lane == 0) red[warp * kLT + lt] = s;
-      }
-      named_sync(1, kWThreads);
-      if (tid < M) {
-        float s = 0.f;
-        for (int qq = 0; qq < 4; ++qq) s += red[((tid & 1) * 4 + qq) * kLT + (tid >> 1)];
-        sl[(size_t)blockIdx.x * kMaxM + tid] = s;
-      }
-      __threadfence();
-      named_sync(1, kWThreads);
-      if (tid == 0) *sflag = atomicAdd(&a.B.ss_counter[a.which], 1u) == (unsigned)(g.P - 1);
-      named_sync(1, kWThreads);
-      if (*sflag) {
-        __threadfence();
-        for (int m = 0; m < M; ++m) {
-          float v = 0.f;
-          for (int b = tid; b < g.P; b += kWThreads) {
-            v += __ldcg(&sl[(size_t)b * kMaxM + m]);
-            if (t_has_split_slot(g, b)) v += __ldcg(&sl[((size_t)kMaxBlocksDev + b) * kMaxM + m]);
-          }
-          v = warp_sum(v);
-          if (lane == 0) red[warp] = v;
-          named_sync(1, kWThreads);
-          if (tid == 0) {
-            float tot = 0.f;
-            for (int w = 0; w < kWorkers; ++w) tot += red[w];
-            a.B.ss[a.which * kMaxM + m] = tot;
-          }
-          named_sync(1, kWThreads);
-        }
-        if (tid == 0) a.B.ss_counter[a.which] = 0u;
-      }
-    } else if constexpr (KIND == kKHead) {
+    // ---- exit head: per-block statistics, and the last block's fixed-order merge
+    if constexpr (KIND == kKHead) {
       HeadPart* sl = static_cast<HeadPart*>(a.B.head_part);
       named_sync(1, kWThreads);
       if (tid < M) {
@@ -668,13 +706,18 @@ __global__ void __launch_bounds__(kTThreads, 1)
       named_sync(1, kWThreads);
       if (*sflag) {
         __threadfence();
+        // per row: every worker thread takes blocks tid, tid + 256, ... (the
+        // running and split slots loaded together), then a shuffle tree per
+        // warp and a tree over the eight warps; the order does not depend on M
         for (int m = 0; m < M; ++m) {
           HeadPart p;
           part_empty(p);
           for (int b = tid; b < g.P; b += kWThreads) {
-            part_merge(p, part_load_cg(&sl[(size_t)b * kMaxM + m]));
-            if (t_has_split_slot(g, b))
-              part_merge(p, part_load_cg(&sl[((size_t)kMaxBlocksDev + b) * kMaxM + m]));
+            const bool sp = t_has_split_slot(g, b);
+            const HeadPart x = part_load_cg(&sl[(size_t)b * kMaxM + m]);
+            const HeadPart y = part_load_cg(&sl[((size_t)kMaxBlocksDev + (sp ? b : 0)) * kMaxM + m]);
+            part_merge(p, x);
+            if (sp) part_merge(p, y);
           }
           for (int off = 16; off > 0; off >>= 1) part_merge(p, part_shfl(p, off));
           if (lane == 0) comb[warp] = p;
@@ -731,7 +774,7 @@ TGeom make_tgeom(const Dims& D, int N, int K, int map) {
     g.ntiles = (N / 2 + 127) / 128;
   else
     g.ntiles = (N + kTR - 1) / kTR;
-  g.T = (long long)g.ntiles * g.nks;
+  g.T = g.ntiles * g.nks;
   g.P = D.num_sms;
   return g;
 }
@@ -739,6 +782,9 @@ TGeom make_tgeom(const Dims& D, int N, int K, int map) {
 template <int TP, int KIND, bool NORM>
 cudaError_t tile_launch(const CUtensorMap& wm, const CUtensorMap& xm, const TArgs& a,
                         cudaStream_t st) {
+  // unit indices are 32-bit: T * blocks must stay below 2^31
+  if (a.g.T < 1 || a.g.T > (1 << 22) || a.g.P < 1 || a.g.P > kMaxBlocksDev)
+    return cudaErrorInvalidValue;
   return launch_ex(k_tile<TP, KIND, NORM>, dim3(a.g.P), dim3(kTThreads),
                    TL<TP, KIND == kKHead>::total, st, wm, xm, a);
 }

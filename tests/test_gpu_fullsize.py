@@ -1,0 +1,191 @@
+"""Parity at the full sizes of the four bf16 decoder shapes (Llama-2-7B,
+Llama-3-8B, Llama-2-13B, Llama-2-70B), with the engine built exactly as the
+benchmark builds it (full weights, the workload's max_seq, the same graphs).
+
+The oracle cannot run these models end to end in seconds, so the checks are
+the ones it can make one output at a time, plus properties that hold at any
+size:
+- weights generated on the device equal the host generator bit for bit on
+  sampled indices of every tensor kind;
+- every projection and the LM head, at M = 1 (drafting) and at M = kmax + 1
+  (a full verification tile), on sampled output rows against the oracle's
+  row-by-row fp64 product of the same generated weights;
+- greedy self-speculative decoding after the workload's full prompt emits
+  exactly the autoregressive tokens, for the seeded LEDE Q-network and for a
+  static (L/2, 4) policy (§3.3 with greedy acceptance, §4.1);
+- exiting at l = L accepts every draft (shared exit head, §3.1.1);
+- Llama-2-7B shape (the benchmark's workload): teacher-forced logits at the
+  exits l = L/2 and l = L within 2e-2 max relative error of the oracle's
+  full model on a short prompt.
+"""
+import gc
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from parity import has_gpu, prompt, rel_err
+from synth.workloads import LLAMA2_7B, LLAMA2_13B, LLAMA2_70B, LLAMA3_8B
+
+pytestmark = [pytest.mark.gpu,
+              pytest.mark.skipif(not has_gpu(), reason="needs a CUDA GPU")]
+
+FULL = {"7b": LLAMA2_7B, "8b": LLAMA3_8B, "13b": LLAMA2_13B, "70b": LLAMA2_70B}
+# new tokens for the invariant runs: the workload's own length where it takes
+# seconds, fewer on the 70B shape (about 20 tokens/s autoregressive)
+GEN = {"7b": 256, "8b": 128, "13b": 96, "70b": 24}
+
+
+@pytest.fixture(scope="module", params=list(FULL))
+def full(request):
+    import torch
+    from paper_2606_03113_gb300.runtime import DeviceModel, Engine
+    w = FULL[request.param]
+    dm = DeviceModel(w.shape)
+    eng = Engine(dm, w.max_seq)
+    yield request.param, w, dm, eng
+    eng.close()
+    del eng, dm
+    gc.collect()
+    torch.cuda.empty_cache()
+
+
+def product_tol(K: int) -> float:
+    """Bound on max |y_gpu - y| / max |y| for a bf16 row times an fp32 input
+    of length K on the tensor cores.  The input enters as bf16 high + low
+    parts, which keep 16 significant bits (error <= 2^-17 per element; 4x
+    that as the bound on the row sum relative to max |y|), and the fp32
+    accumulator takes one 16-wide block of products per step, each addition
+    correct to 1 ulp (2^-23) of the running sum, so K/16 additions add at
+    most (K/16) 2^-23 (a worst case: errors are taken to share a sign, as
+    with truncating hardware adders).  For K = 4096 this is 6.1e-5; the
+    measured errors at full size are 2e-6 to 1.5e-5."""
+    return 4 * 2.0 ** -17 + (K / 16) * 2.0 ** -23
+
+
+def _sample_rows(n: int, rng) -> np.ndarray:
+    mid = int(rng.integers(64, max(65, n - 128)))
+    return np.unique(np.r_[0:32, mid:mid + 32, n - 32:n])
+
+
+def test_weights_bitwise_sampled(full):
+    name, w, dm, eng = full
+    s = w.shape
+    rng = np.random.default_rng(7)
+    L = s.n_layers
+    cases = [(dm.embed, synth.TID_EMBED, s.sigma), (dm.lm_head, synth.TID_LMHEAD, s.sigma)]
+    for l in (0, L // 2 - 1, L // 2, L - 1):
+        late = s.late_scale if l >= L // 2 else 1.0
+        base = synth.layer_tid(l, 0)
+        cases += [(dm.layers[l]["wqkv"], base + 0, s.sigma),
+                  (dm.layers[l]["wo"], base + 1, s.sigma * late),
+                  (dm.layers[l]["w_gate_up"], base + 2, s.sigma),
+                  (dm.layers[l]["w_down"], base + 3, s.sigma * late)]
+    for t, tid, sig in cases:
+        flat = t.view(-1)
+        n = flat.numel()
+        for start in (0, int(rng.integers(0, n - 4096)), n - 4096):
+            g = flat[start:start + 4096].view(dtype=__import__("torch").int16).cpu().numpy()
+            ref = synth.weights_bf16_bits(synth.SEED_WEIGHTS, tid, start, 4096, sig)
+            assert np.array_equal(g.view(np.uint16), ref), (name, tid, start)
+
+
+@pytest.mark.parametrize("M", [1, "kmax+1"])
+def test_projections_sampled_rows(full, M):
+    import torch
+    name, w, dm, eng = full
+    s = w.shape
+    M = 1 if M == 1 else w.kmax + 1
+    rng = np.random.default_rng(11 + M)
+    L = s.n_layers
+    qd = s.n_heads * s.head_dim
+    mats = []  # (which, layer, rows, cols, tid, sigma)
+    for l in (0, L - 1):
+        late = s.late_scale if l >= L // 2 else 1.0
+        base = synth.layer_tid(l, 0)
+        mats += [(0, l, s.qkv_rows, s.d_model, base + 0, s.sigma),
+                 (1, l, s.d_model, qd, base + 1, s.sigma * late),
+                 (2, l, 2 * s.ffn_dim, s.d_model, base + 2, s.sigma),
+                 (3, l, s.d_model, s.ffn_dim, base + 3, s.sigma * late)]
+    mats.append((4, 0, s.vocab, s.d_model, synth.TID_LMHEAD, s.sigma))
+    cols_of = {which: cols for which, _, _, cols, _, _ in mats}
+    errs = []
+    for which, layer, rows, cols, tid, sig in mats:
+        x = rng.normal(size=(M, cols)).astype(np.float32)
+        xd = torch.from_numpy(x).cuda()
+        yd = torch.full((M, rows), float("nan"), dtype=torch.float32, device="cuda")
+        eng.op_gemv(which, layer, xd, yd)
+        torch.cuda.synchronize()
+        y = yd.cpu().numpy()
+        assert np.isfinite(y).all(), (name, which, layer)
+        sel = _sample_rows(rows, rng)
+        for m in sorted({0, M // 2, M - 1}):
+            ref = np.empty(sel.size)
+            # contiguous runs of sampled rows, each one oracle call
+            runs = np.split(sel, np.where(np.diff(sel) != 1)[0] + 1)
+            off = 0
+            for r in runs:
+                ref[off:off + r.size] = oracle.matvec_synth(synth.SEED_WEIGHTS, tid, sig, True,
+                                                            int(r[0]), r.size,
+                                                            x[m].astype(np.float64))
+                off += r.size
+            errs.append((which, layer, m, rel_err(y[m, sel], ref)))
+    print(name, M, ["%d/%d/%d: %.2e" % e for e in errs])
+    bad = [e for e in errs if not e[3] < product_tol(cols_of[e[0]])]
+    assert not bad, (name, M, bad)
+
+
+def test_ssd_equals_ar_after_full_prompt(full):
+    name, w, dm, eng = full
+    L = w.shape.n_layers
+    n = GEN[name]
+    ids = prompt(w)
+    eng.set_ar()
+    eng.prefill(ids)
+    ar, _, _ = eng.generate(n)
+    eng.set_lede(w, synth.qnet_hidden_params(3, w.qnet_hidden))
+    eng.prefill(ids)
+    le, nr, _ = eng.generate(n)
+    assert np.array_equal(ar, le), name
+    tr = eng.traces(nr)
+    assert sum(t["n_emit"] for t in tr) == n
+    eng.set_static(L // 2, 4, kmax=w.kmax)
+    eng.prefill(ids)
+    st, _, _ = eng.generate(n)
+    assert np.array_equal(ar, st), name
+
+
+def test_full_depth_exit_accepts_every_draft(full):
+    name, w, dm, eng = full
+    L = w.shape.n_layers
+    eng.set_static(L, 4, kmax=4)
+    eng.prefill(prompt(w))
+    _, nr, _ = eng.generate(min(40, GEN[name]))
+    tr = eng.traces(nr)
+    assert all(t["a"] == t["k"] and t["lstar"] == L for t in tr if t["kcap"] > 0)
+
+
+def test_teacher_forced_logits_full_7b(full):
+    name, w, dm, eng = full
+    if name != "7b":
+        pytest.skip("the oracle's full-model forward is run on the benchmark's shape only")
+    s = w.shape
+    ids = prompt(w, 12)
+    n0 = 8
+    om = oracle.Model(s)
+    try:
+        sess = om.session(64)
+        eng.set_ar()
+        eng.prefill(ids[:n0])
+        for l_exit in (s.n_layers // 2, s.n_layers):
+            z, st = eng.forward_exit(ids[n0:], n0, l_exit)
+            h = sess.forward(ids, 0, 0, l_exit)
+            for i in range(len(ids) - n0):
+                zr, sr = om.exit_head(h[n0 + i])
+                assert rel_err(z[i], zr) < 2e-2, (l_exit, i, rel_err(z[i], zr))
+                if sr["margin"] > 5e-2:
+                    assert st[i]["argmax"] == sr["argmax"], (l_exit, i)
+                assert abs(st[i]["entropy"] - sr["entropy"]) <= 2e-2 * max(1.0, sr["entropy"])
+    finally:
+        om.close()
