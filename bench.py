@@ -194,7 +194,7 @@ def time_generate(eng, ids, n_new, dist_barrier) -> tuple:
     return e0.elapsed_time(e1), ne, tr
 
 
-KERNEL_NAMES = {0: "k_qkv", 1: "k_attn+k_attn_combine", 2: "k_resid(wo)", 3: "k_gate_up",
+KERNEL_NAMES = {0: "k_qkv", 1: "k_attn", 2: "k_resid(wo)", 3: "k_gate_up",
                 4: "k_resid(w_down)", 5: "k_head"}
 
 

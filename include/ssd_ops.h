@@ -59,8 +59,8 @@ ssd_status ssd_op_gemv(ssd_ctx* ctx, int32_t which, int32_t layer, int32_t M, co
 
 /* One launch of one hot-path kernel of layer `layer` exactly as the round
  * graphs launch it, on M rows at positions pos0..pos0+M-1 of the context's
- * own buffers: kernel = 0 QKV (+RoPE, KV append), 1 attention (split-K and
- * combine), 2 O projection (+residual), 3 gate/up (+RMSNorm, SwiGLU),
+ * own buffers: kernel = 0 QKV (+RoPE, KV append), 1 attention (split-K with
+ * the split merge in the same kernel), 2 O projection (+residual), 3 gate/up (+RMSNorm, SwiGLU),
  * 4 down projection (+residual), 5 exit head (final RMSNorm, LM head,
  * statistics; layer ignored).  It overwrites the activations and the KV rows
  * at those positions: for timing and profiling, not inside a generation.

@@ -1,14 +1,25 @@
 // attention.cu -- split-K decode attention over the contiguous KV cache for
-// 1 (drafting, AR) or k + 1 (verification) query rows, with GQA.
+// 1 (drafting, autoregressive) or k + 1 (verification) query rows, with GQA,
+// in one kernel.
 //
-// Grid = (key splits of 32, KV heads).  A block stages its 32 keys and values
-// once (converted to fp32 in shared memory) and serves every query head of
-// the KV group and every query row with them, so a GQA group of G heads and M
-// rows share one KV read.  Row m sits at position pos0 + m and attends
-// causally to keys [0, pos0 + m] (the new rows' own keys were appended by the
-// QKV kernel).  Each (row, head, split) writes an unnormalised partial
-// (max, sum, output); the combine kernel merges splits with the log-sum-exp
-// rule.
+// Grid = (key splits of kAttnKeys, KV heads).  A block stages its keys and
+// values once (fp32 in shared memory) and serves every query head of the KV
+// group and every query row with them, so a GQA group of G heads and M rows
+// share one KV read.  Row m sits at position pos0 + m and attends causally to
+// keys [0, pos0 + m] (the new rows' own keys were appended by the QKV kernel).
+//
+// Keys before pos0 were written by earlier passes, so a block loads them
+// before waiting for the QKV kernel that precedes it (programmatic dependent
+// launch) and loads only the M new keys after the wait.  The row window
+// (pos0, M) is read before the wait too: every writer of the control block
+// runs at least one full dependency before this kernel is launched; it is
+// read again after the wait and a mismatch is flagged and handled by
+// reloading every key.
+//
+// Each (row, head, split) writes an unnormalised partial (max, sum, output);
+// the last split block to finish a (KV head, row) pair -- a ticket per pair --
+// merges its G heads' partials in split order with the log-sum-exp rule, so
+// the result does not depend on which block finishes last.
 #include <math.h>
 
 #include "kernels.h"
@@ -16,78 +27,134 @@
 
 namespace ssd {
 
-template <typename T, int MM>
-__global__ void __launch_bounds__(kWarps * 32) k_attn(Dims D, Bufs B, int layer, RowSel sel) {
+namespace {
+
+constexpr int kAK = kAttnKeys;   // keys per split (two per lane)
+constexpr int kAThreads = 256;
+constexpr int kAWarps = kAThreads / 32;
+
+// Stages keys [k0, k1) of the split (relative to s0) into shared memory:
+// all global loads are issued before any is converted.
+template <typename T>
+__device__ __forceinline__ void stage_keys(const T* kb, const T* vb, int hd, int k0, int k1,
+                                           float* Ks, float* Vs) {
+  using E = Elem<T>;
+  constexpr int EPC = E::kPerChunk;
+  const int cpr = hd / EPC;  // 16-byte chunks per key row
+  const int n = (k1 - k0) * cpr;
+  constexpr int kUnroll = 4;
+  for (int c0 = threadIdx.x; c0 < n; c0 += kAThreads * kUnroll) {
+    uint4 ku[kUnroll], vu[kUnroll];
+#pragma unroll
+    for (int j = 0; j < kUnroll; ++j) {
+      const int c = c0 + j * kAThreads;
+      if (c < n) {
+        const int key = k0 + c / cpr, off = (c % cpr) * EPC;
+        ku[j] = __ldg(reinterpret_cast<const uint4*>(kb + (size_t)key * hd + off));
+        vu[j] = __ldg(reinterpret_cast<const uint4*>(vb + (size_t)key * hd + off));
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < kUnroll; ++j) {
+      const int c = c0 + j * kAThreads;
+      if (c < n) {
+        const int key = k0 + c / cpr, off = (c % cpr) * EPC;
+        float kf[EPC], vf[EPC];
+        E::unpack(ku[j], kf);
+        E::unpack(vu[j], vf);
+#pragma unroll
+        for (int e = 0; e < EPC; ++e) {
+          Ks[key * (hd + 1) + off + e] = kf[e];
+          Vs[key * hd + off + e] = vf[e];
+        }
+      }
+    }
+  }
+}
+
+}  // namespace
+
+template <typename T>
+__global__ void __launch_bounds__(kAThreads) k_attn(Dims D, Bufs B, int layer, RowSel sel) {
   extern __shared__ float sm[];
   const int split = blockIdx.x, g = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  pdl_wait();
-  pdl_launch_dependents();
-  int pos0, M;
-  resolve_rows(B.ctl, sel, pos0, M);
-  const int s0 = split * kAttnChunk;
-  if (s0 > pos0 + M - 1) return;  // beyond every row's causal window
   const int hd = D.hd;
-  float* Ks = sm;                         // [32][hd + 1] (padded: lane-per-key reads)
-  float* Vs = Ks + kAttnChunk * (hd + 1); // [32][hd]
-  float* Ps = Vs + kAttnChunk * hd;       // [kWarps][32]
-  using E = Elem<T>;
-  constexpr int EPC = E::kPerChunk;
+  const int G = D.Hq / D.Hkv;
+  float* Ks = sm;                           // [kAK][hd + 1] (padded: lane-per-key reads)
+  float* Vs = Ks + kAK * (hd + 1);          // [kAK][hd]
+  float* Ps = Vs + kAK * hd;                // [warps][kAK] probabilities
+  float* Cw = Ps + kAWarps * kAK;           // merge: [G][nsplit] sums, then weights
+  float* Cm = Cw + (size_t)G * D.nsplit;    // merge: [G][nsplit] maxima
+  float* CL = Cm + (size_t)G * D.nsplit;    // merge: [G] denominators
+  int* last_rows = reinterpret_cast<int*>(CL + G);  // [kMaxM] rows this block merges
+  __shared__ int s_nlast;
+
   const T* kv = static_cast<const T*>(B.kv) + (size_t)layer * 2 * D.Hkv * D.max_seq * hd;
+  const int s0 = split * kAK;
   const T* kb = kv + ((size_t)g * D.max_seq + s0) * hd;
   const T* vb = kv + ((size_t)(D.Hkv + g) * D.max_seq + s0) * hd;
-  const int cpr = hd / EPC;  // chunks per key row
-  const int nkeys = min(kAttnChunk, pos0 + M - s0);
-  for (int c = threadIdx.x; c < kAttnChunk * cpr; c += blockDim.x) {
-    const int key = c / cpr, off = (c - key * cpr) * EPC;
-    float kf[EPC], vf[EPC];
-    if (key < nkeys) {
-      E::unpack(__ldg(reinterpret_cast<const uint4*>(kb + (size_t)key * hd + off)), kf);
-      E::unpack(__ldg(reinterpret_cast<const uint4*>(vb + (size_t)key * hd + off)), vf);
-    } else {
-#pragma unroll
-      for (int e = 0; e < EPC; ++e) kf[e] = vf[e] = 0.f;
-    }
-#pragma unroll
-    for (int e = 0; e < EPC; ++e) {
-      Ks[key * (hd + 1) + off + e] = kf[e];
-      Vs[key * hd + off + e] = vf[e];
+
+  // keys written by earlier passes: loaded before the wait
+  int pos0, M;
+  resolve_rows(B.ctl, sel, pos0, M);
+  int nold = min(max(min(pos0, D.max_seq) - s0, 0), kAK);  // clamped: never past the cache
+  if (pos0 + M > s0 && nold > 0) stage_keys<T>(kb, vb, hd, 0, nold, Ks, Vs);
+  pdl_wait();
+  pdl_launch_dependents();
+  {
+    int p2, m2;
+    resolve_rows(B.ctl, sel, p2, m2);
+    if (p2 != pos0 || m2 != M) {  // the window moved: reload every key
+      if (threadIdx.x == 0) atomicOr(&B.ctl->err, (int)kErrControl);
+      pos0 = p2;
+      M = m2;
+      nold = 0;
     }
   }
+  if (s0 > pos0 + M - 1) return;  // beyond every row's causal window
+  const int nkeys = min(kAK, pos0 + M - s0);
+  if (nkeys > nold) stage_keys<T>(kb, vb, hd, nold, nkeys, Ks, Vs);
   __syncthreads();
-  const int G = D.Hq / D.Hkv;
+
+  // partial attention of every (row, head) pair of the group over this split
   const float scale = 1.0f / sqrtf((float)hd);
-  float* pw = Ps + warp * kAttnChunk;
-  for (int gm = warp; gm < G * M; gm += kWarps) {
-    const int m = gm / G, qh = g * G + (gm - m * G);
+  float* pw = Ps + warp * kAK;
+  const int m_first = max(0, s0 - pos0);  // rows that see at least one key here
+  const int npairs = G * (M - m_first);
+  for (int pi = warp; pi < npairs; pi += kAWarps) {
+    const int m = m_first + pi / G, qh = g * G + pi % G;
     const int pos = pos0 + m;
     const float* q = B.xq + (size_t)m * D.qd + (size_t)qh * hd;
-    const int key = s0 + lane;
-    const bool valid = key <= pos;
-    float sc = -INFINITY;
-    if (valid) {
-      float dot = 0.f;
-      const float* kr = Ks + lane * (hd + 1);
-      for (int i = 0; i < hd; i += 4) {
-        const float4 qv = __ldg(reinterpret_cast<const float4*>(q + i));
-        dot = fmaf(qv.x, kr[i], dot);
-        dot = fmaf(qv.y, kr[i + 1], dot);
-        dot = fmaf(qv.z, kr[i + 2], dot);
-        dot = fmaf(qv.w, kr[i + 3], dot);
-      }
-      sc = dot * scale;
+    const int ka = lane, kb2 = lane + 32;
+    const bool va = s0 + ka <= pos && ka < nkeys, vb2 = s0 + kb2 <= pos && kb2 < nkeys;
+    float da = 0.f, db = 0.f;
+    const float* kra = Ks + ka * (hd + 1);
+    const float* krb = Ks + kb2 * (hd + 1);
+    for (int i = 0; i < hd; i += 4) {
+      const float4 qv = __ldg(reinterpret_cast<const float4*>(q + i));
+      da = fmaf(qv.x, kra[i], da);
+      da = fmaf(qv.y, kra[i + 1], da);
+      da = fmaf(qv.z, kra[i + 2], da);
+      da = fmaf(qv.w, kra[i + 3], da);
+      db = fmaf(qv.x, krb[i], db);
+      db = fmaf(qv.y, krb[i + 1], db);
+      db = fmaf(qv.z, krb[i + 2], db);
+      db = fmaf(qv.w, krb[i + 3], db);
     }
-    const float mx = warp_max(sc);
-    const float p = valid ? expf(sc - mx) : 0.f;
-    const float l = warp_sum(p);
-    pw[lane] = p;
+    const float sa = va ? da * scale : -INFINITY, sb = vb2 ? db * scale : -INFINITY;
+    const float mx = warp_max(fmaxf(sa, sb));
+    const float pa = va ? expf(sa - mx) : 0.f, pb = vb2 ? expf(sb - mx) : 0.f;
+    const float l = warp_sum(pa + pb);
+    pw[ka] = pa;
+    pw[kb2] = pb;
     __syncwarp();
     const size_t pidx = ((size_t)m * D.Hq + qh) * D.nsplit + split;
     float* part = B.attn_part + pidx * hd;
     for (int dd = lane; dd < hd; dd += 32) {
       float o = 0.f;
 #pragma unroll 8
-      for (int s = 0; s < kAttnChunk; ++s) o = fmaf(pw[s], Vs[s * hd + dd], o);
+      for (int s = 0; s < nkeys; ++s) o = fmaf(pw[s], Vs[s * hd + dd], o);
       part[dd] = o;
     }
     if (lane == 0) {
@@ -96,62 +163,96 @@ __global__ void __launch_bounds__(kWarps * 32) k_attn(Dims D, Bufs B, int layer,
     }
     __syncwarp();
   }
-}
 
-// out[m][qh*hd + d] = sum_s e^{m_s - M} o_s[d] / sum_s e^{m_s - M} l_s over the
-// splits that hold keys of row m.
-template <int MM>
-__global__ void k_attn_combine(Dims D, Bufs B, RowSel sel) {
-  const int qh = blockIdx.x, m = blockIdx.y;
-  pdl_wait();
-  pdl_launch_dependents();
-  int pos0, M;
-  resolve_rows(B.ctl, sel, pos0, M);
-  if (m >= M) return;
-  const int nsp = (pos0 + m) / kAttnChunk + 1;
-  const size_t base = ((size_t)m * D.Hq + qh) * D.nsplit;
-  float gmax = -INFINITY;
-  for (int s = 0; s < nsp; ++s) gmax = fmaxf(gmax, B.attn_ml[2 * (base + s)]);
-  for (int dd = threadIdx.x; dd < D.hd; dd += blockDim.x) {
-    float L = 0.f, O = 0.f;
-    for (int s = 0; s < nsp; ++s) {
-      const float l = B.attn_ml[2 * (base + s) + 1];
-      if (l > 0.f) {
-        const float w = expf(B.attn_ml[2 * (base + s)] - gmax);
-        L = fmaf(w, l, L);
-        O = fmaf(w, B.attn_part[(base + s) * D.hd + dd], O);
-      }
+  // tickets: the last split of (g, m) merges the group's heads for row m
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_nlast = 0;
+  __syncthreads();
+  if (threadIdx.x < M && threadIdx.x >= m_first) {
+    const int m = threadIdx.x;
+    const int nsp = (pos0 + m) / kAK + 1;
+    uint32_t* cnt = B.attn_counter + (size_t)g * kMaxM + m;
+    if (atomicAdd(cnt, 1u) == (uint32_t)(nsp - 1)) {
+      *cnt = 0u;
+      last_rows[atomicAdd(&s_nlast, 1)] = m;
     }
-    B.attn_out[(size_t)m * D.qd + (size_t)qh * D.hd + dd] = O / L;
+  }
+  __syncthreads();
+  const int nlast = s_nlast;
+  if (nlast == 0) return;
+  __threadfence();
+  for (int li = 0; li < nlast; ++li) {
+    const int m = last_rows[li];
+    const int nsp = (pos0 + m) / kAK + 1;
+    const size_t hbase = ((size_t)m * D.Hq + (size_t)g * G) * D.nsplit;
+    // (max, sum) of every head and split: one round of loads into shared memory
+    for (int i = threadIdx.x; i < G * nsp; i += kAThreads) {
+      const int h = i / nsp, s = i - h * nsp;
+      const size_t pidx = hbase + (size_t)h * D.nsplit + s;
+      Cm[h * D.nsplit + s] = __ldcg(&B.attn_ml[2 * pidx]);
+      Cw[h * D.nsplit + s] = __ldcg(&B.attn_ml[2 * pidx + 1]);
+    }
+    __syncthreads();
+    // weights e^{m_s - max} and denominators (one warp per head, fixed lane order)
+    for (int h = warp; h < G; h += kAWarps) {
+      float gmax = -INFINITY;
+      for (int s = lane; s < nsp; s += 32) gmax = fmaxf(gmax, Cm[h * D.nsplit + s]);
+      gmax = warp_max(gmax);
+      float L = 0.f;
+      for (int s = lane; s < nsp; s += 32) {
+        const float l = Cw[h * D.nsplit + s];
+        const float w = l > 0.f ? expf(Cm[h * D.nsplit + s] - gmax) : 0.f;
+        Cw[h * D.nsplit + s] = w;
+        L = fmaf(w, l, L);
+      }
+      L = warp_sum(L);
+      if (lane == 0) CL[h] = L;
+    }
+    __syncthreads();
+    // outputs: partials of eight splits loaded per round, added in split order
+    for (int o = threadIdx.x; o < G * hd; o += kAThreads) {
+      const int h = o / hd, dd = o - h * hd;
+      const float* part = B.attn_part + (hbase + (size_t)h * D.nsplit) * hd + dd;
+      const float* w = Cw + h * D.nsplit;
+      float O = 0.f;
+      for (int sc = 0; sc < nsp; sc += 8) {
+        float pv[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) pv[j] = sc + j < nsp ? __ldcg(part + (size_t)(sc + j) * hd) : 0.f;
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          if (sc + j < nsp) O = fmaf(w[sc + j], pv[j], O);
+      }
+      B.attn_out[(size_t)m * D.qd + (size_t)(g * G + h) * hd + dd] = O / CL[h];
+    }
+    __syncthreads();
   }
 }
 
-static size_t attn_smem(int hd) {
-  return sizeof(float) * ((size_t)kAttnChunk * (hd + 1) + (size_t)kAttnChunk * hd +
-                          (size_t)kWarps * kAttnChunk);
+size_t attn_smem(const Dims& D) {
+  const int G = D.Hq / D.Hkv;
+  return sizeof(float) * ((size_t)kAK * (D.hd + 1) + (size_t)kAK * D.hd + (size_t)kAWarps * kAK +
+                          2 * (size_t)G * D.nsplit + G) +
+         sizeof(int) * kMaxM;
 }
 
-template <typename T, int MM>
+template <typename T>
 static cudaError_t attn_t(const Dims& D, const Bufs& B, int layer, RowSel sel, cudaStream_t st) {
   dim3 grid(D.nsplit, D.Hkv);
-  const size_t smem = attn_smem(D.hd);
+  const size_t smem = attn_smem(D);
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(k_attn<T, MM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+    cudaError_t e =
+        cudaFuncSetAttribute(k_attn<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
   }
-  cudaError_t e = launch_ex(k_attn<T, MM>, grid, dim3(kWarps * 32), smem, st, D, B, layer, sel);
-  if (e != cudaSuccess) return e;
-  return launch_ex(k_attn_combine<MM>, dim3(D.Hq, MM), dim3(D.hd < 128 ? D.hd : 128), 0, st, D, B,
-                   sel);
+  return launch_ex(k_attn<T>, grid, dim3(kAThreads), smem, st, D, B, layer, sel);
 }
 
 cudaError_t launch_attention(const Dims& D, const Bufs& B, int dtype, int layer, RowSel sel,
-                             bool big, cudaStream_t st) {
-  if (dtype == SSD_DTYPE_BF16)
-    return big ? attn_t<__nv_bfloat16, kMaxM>(D, B, layer, sel, st)
-               : attn_t<__nv_bfloat16, 1>(D, B, layer, sel, st);
-  return big ? attn_t<float, kMaxM>(D, B, layer, sel, st) : attn_t<float, 1>(D, B, layer, sel, st);
+                             bool /*big*/, cudaStream_t st) {
+  if (dtype == SSD_DTYPE_BF16) return attn_t<__nv_bfloat16>(D, B, layer, sel, st);
+  return attn_t<float>(D, B, layer, sel, st);
 }
 
 }  // namespace ssd

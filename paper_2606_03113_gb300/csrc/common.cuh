@@ -18,8 +18,8 @@ constexpr int kMaxCand = SSD_TRACE_MAXC;
 constexpr int kTraceCap = 64;      // C_trace window capacity
 constexpr int kTopK = 8;           // max k of the token confidence
 constexpr int kWarps = 8;          // warps per block of the matrix-vector kernels
-constexpr int kAttnChunk = 32;     // keys per attention split (one per lane)
-constexpr int kLayerKernels = 6;   // qkv, attention, combine, o, gate/up, down
+constexpr int kAttnKeys = 64;      // keys per attention split (two per lane)
+constexpr int kLayerKernels = 5;   // launches per layer: qkv, attention, o, gate/up, down
 
 // Which rows a kernel works on.  Inside the round graphs they follow the
 // device control block; prefill and the op entry points pass them directly.
@@ -161,6 +161,7 @@ struct Bufs {
   float* xq;         // [kMaxM][qd] rotated queries
   float* attn_part;  // [kMaxM][Hq][nsplit][hd] unnormalised partial outputs
   float* attn_ml;    // [kMaxM][Hq][nsplit][2] partial (max, sum)
+  uint32_t* attn_counter;  // [Hkv][kMaxM] split tickets of the attention merge
   float* attn_out;   // [kMaxM][qd]
   float* act;        // [kMaxM][F]
   float* logits;     // [kMaxM][V] (written only when requested)

@@ -56,7 +56,7 @@ size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
   d.max_seq = c.max_seq;
   d.qd = c.n_heads * c.head_dim;
   d.kvd = c.n_kv_heads * c.head_dim;
-  d.nsplit = (c.max_seq + kAttnChunk - 1) / kAttnChunk;
+  d.nsplit = (c.max_seq + kAttnKeys - 1) / kAttnKeys;
   d.eps = c.rms_eps;
   d.num_sms = kMaxBlocks;  // set to the device's SM count at init
   d.ss_tiles = (c.d_model + 15) / 16;
@@ -80,6 +80,7 @@ size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
   b.xq = cv.take<float>(sizeof(float) * kMaxM * d.qd);
   b.attn_part = cv.take<float>(sizeof(float) * kMaxM * d.Hq * (size_t)d.nsplit * d.hd);
   b.attn_ml = cv.take<float>(sizeof(float) * kMaxM * d.Hq * (size_t)d.nsplit * 2);
+  b.attn_counter = cv.take<uint32_t>(sizeof(uint32_t) * (size_t)d.Hkv * kMaxM);
   b.attn_out = cv.take<float>(sizeof(float) * kMaxM * d.qd);
   b.act = cv.take<float>(sizeof(float) * kMaxM * d.F);
   b.logits = cv.take<float>(sizeof(float) * kMaxM * (size_t)d.V);
@@ -499,6 +500,8 @@ ssd_status ssd_init_model(const ssd_model_cfg* cfg, const ssd_weights* w, void* 
   if (e == cudaSuccess)
     e = cudaMemsetAsync(x->B.ss_part, 0, sizeof(float) * 2 * (size_t)x->D.ss_nt * kMaxM, x->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(x->B.ss_counter, 0, sizeof(uint32_t) * 2, x->stream);
+  if (e == cudaSuccess)
+    e = cudaMemsetAsync(x->B.attn_counter, 0, sizeof(uint32_t) * (size_t)x->D.Hkv * kMaxM, x->stream);
   if (e == cudaSuccess)
     e = cudaMemsetAsync(x->B.tile_counter, 0, sizeof(uint32_t) * (size_t)x->D.max_tiles, x->stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(x->stream);

@@ -918,7 +918,7 @@ cudaError_t launch_layer_part(const Dims& D, const Bufs& B, int dtype, const Lay
 
 cudaError_t launch_layer(const Dims& D, const Bufs& B, int dtype, const LayerW& w,
                          const TileMaps* tm, int layer, RowSel sel, int mrows, cudaStream_t st) {
-  for (int part = 0; part < kLayerKernels - 1; ++part) {
+  for (int part = 0; part < 5; ++part) {  // qkv, attention, o, gate/up, down
     cudaError_t e = launch_layer_part(D, B, dtype, w, tm, layer, part, sel, mrows, st);
     if (e != cudaSuccess) return e;
   }

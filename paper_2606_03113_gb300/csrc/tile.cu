@@ -551,11 +551,11 @@ __global__ void __launch_bounds__(kTThreads, 1)
 #pragma unroll
       for (int lt = 0; lt < LTN; ++lt) u0[lt] = u1[lt] = 0.f;
       if (M == 1) {
-        // one token (drafting, autoregressive steps): eight contributors per round
-        for (int b = grp == 0 ? b0 : b1 + 1; b <= b1; b += 8) {
-          float c0[8], c1[8];
+        // one token (drafting, autoregressive steps): sixteen contributors per round
+        for (int b = grp == 0 ? b0 : b1 + 1; b <= b1; b += 16) {
+          float c0[16], c1[16];
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
+          for (int j = 0; j < 16; ++j) {
             const int bb = b + j;
             bool use = false;
             int sl = 0;
@@ -571,7 +571,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
             c1[j] = use ? x1 : 0.f;
           }
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
+          for (int j = 0; j < 16; ++j) {
             u0[0] += c0[j];
             u1[0] += c1[j];
           }

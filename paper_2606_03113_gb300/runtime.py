@@ -183,9 +183,9 @@ class Engine:
 
 def kernels_per_round(trace: dict, n_layers: int, kind: int) -> int:
     """Kernel launches of one round of the round graph, from its record:
-    round_begin, walk (embed, 6 per layer, head, decide per visited segment),
-    draft_begin, drafts (embed, 6 per layer, head, decide), verify (embed,
-    6 per layer, head), accept."""
+    round_begin, walk (embed, 5 per layer, head, decide per visited segment),
+    draft_begin, drafts (embed, 5 per layer, head, decide), verify (embed,
+    5 per layer, head), accept."""
     per_layer = S.KERNELS_PER_LAYER
     n = 1  # round_begin
     if trace["kcap"] > 0:

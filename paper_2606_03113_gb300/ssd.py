@@ -22,7 +22,7 @@ SSD_DTYPE_F32, SSD_DTYPE_BF16 = 0, 1
 SSD_POLICY_AR, SSD_POLICY_STATIC, SSD_POLICY_LEDE = 0, 1, 2
 TRACE_MAXK, TRACE_MAXQ, TRACE_MAXC = 16, 48, 16
 MAX_M = 17
-KERNELS_PER_LAYER = 6
+KERNELS_PER_LAYER = 5
 
 
 class ssd_model_cfg(C.Structure):
