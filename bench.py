@@ -13,8 +13,10 @@ Prints one JSON line.  --impl reference times the CPU oracle instead.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -42,6 +44,31 @@ def measured_peaks() -> dict:
         d = json.load(open(p))
         return dict(hbm_gbs=float(d["hbm_gbs"]), src="measured")
     return dict(hbm_gbs=6800.0, src="fallback")
+
+
+# DRAM traffic of the dominant kernel from the committed ncu summary: valid
+# only while the kernel's sources are the ones that were captured.
+TRAFFIC_PROFILE = os.path.join(REPO, "profiles", "k_tile_gate_up_llama2-7b.md")
+TRAFFIC_SOURCES = ("tile.cu", "tc.cuh", "pipe.cuh", "headpart.cuh")
+
+
+def measured_traffic() -> int | None:
+    """DRAM read + write bytes per single-row gate/up launch (Llama-2-7B
+    shape) from one ncu capture, or None when the summary is missing or the
+    kernel sources no longer hash to the captured value."""
+    try:
+        text = open(TRAFFIC_PROFILE).read()
+        h = hashlib.sha256()
+        for f in TRAFFIC_SOURCES:
+            with open(os.path.join(REPO, "paper_2606_03113_gb300", "csrc", f), "rb") as fh:
+                h.update(fh.read())
+    except OSError:
+        return None
+    digest = re.search(r"`([0-9a-f]{64})`", text)
+    nbytes = re.search(r"dram bytes per launch \(M = 1\): (\d+)", text)
+    if not digest or not nbytes or digest.group(1) != h.hexdigest():
+        return None
+    return int(nbytes.group(1))
 
 
 # --------------------------------------------------------------- bytes model
@@ -365,8 +392,9 @@ def main():
 
     roof = kernel_roofline(eng, w, peak, pos0=w.prompt_len + n_new // 2)
     dom = max(roof.items(), key=lambda kv: kv[1]["us"] * kv[1]["launches_per_forward"])
+    traffic = measured_traffic() if (w.name == "llama2-7b" and dom[0] == "k_gate_up") else None
     roofline = dict(bound="hbm", achieved=dom[1]["gbs"], peak=peak, unit="GB/s",
-                    frac=dom[1]["gbs"] / peak, traffic=None,
+                    frac=dom[1]["gbs"] / peak, traffic=traffic,
                     kernel=f"{dom[0]} single-row ({dom[1]['bytes'] / 1e6:.1f} MB per launch)",
                     peak_source=f"{peaks['src']} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
                     kernels=roof,
