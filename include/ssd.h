@@ -78,13 +78,27 @@ typedef struct {
   const void* const* w_down;      /* [d_model][ffn_dim] */
 } ssd_weights;
 
-typedef enum { SSD_POLICY_AR = 0, SSD_POLICY_STATIC = 1, SSD_POLICY_LEDE = 2 } ssd_policy_kind;
+typedef enum {
+  SSD_POLICY_AR = 0,
+  SSD_POLICY_STATIC = 1,
+  SSD_POLICY_LEDE = 2,
+  SSD_POLICY_THRESHOLD = 3
+} ssd_policy_kind;
 
-/* Speculation policy.
- *  AR:     plain greedy decoding with the full model (one token per round).
- *  STATIC: fixed exit layer static_l and draft length static_k (LayerSkip).
- *  LEDE:   Q-network over candidate exit layers cand_layers[0..n_cand), ascending
- *          in 1..n_layers; forced exit at the last one; adaptive drafting.
+/* Speculation policy (§3.3 and the baselines and ablations of §4.1, Table 3).
+ *  AR:        plain greedy decoding with the full model (one token per round).
+ *  STATIC:    fixed exit layer static_l and draft length static_k (LayerSkip).
+ *  LEDE:      Q-network over candidate exit layers cand_layers[0..n_cand),
+ *             ascending in 1..n_layers; forced exit at the last one; adaptive
+ *             drafting.  n_cand = 1 is the ablation without dynamic exit
+ *             (exit layer fixed, drafting still decided by the Q-network);
+ *             fixed_k > 0 is the ablation without adaptive drafting (the walk
+ *             picks l*, then exactly min(fixed_k, cap) tokens are drafted and
+ *             the Q-network is not consulted after a draft).
+ *  THRESHOLD: fixed exit layer static_l; after each draft, drafting goes on
+ *             while that draft's max-probability is >= conf_threshold, up to
+ *             kmax (a Draft & Verify-style confidence rule with a fixed
+ *             threshold).
  * kmax caps the drafts per round (1..16).  qnet_params (host fp32, copied) packs
  * W1[qnet_hidden][3], b1[qnet_hidden], W2[2][qnet_hidden], b2[2]; output 0 is
  * Q(continue), output 1 is Q(exit); ties pick continue. */
@@ -98,6 +112,8 @@ typedef struct {
   const float* qnet_params;
   int32_t trace_T; /* C_trace window, 1..64 (paper: 20) */
   int32_t topk;    /* k of the token confidence, 1..8 (paper: 5) */
+  int32_t fixed_k; /* LEDE: 0 = adaptive drafting; 1..16 = fixed draft length */
+  float conf_threshold; /* THRESHOLD: (0, 1] */
 } ssd_policy;
 
 typedef struct {

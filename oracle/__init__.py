@@ -20,7 +20,7 @@ BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(BUILD_DIR, "liboracle.so")
 
 MAX_CAND, MAX_K, MAX_Q, TOPK_MAX = 32, 32, 64, 8
-POLICY_AR, POLICY_STATIC, POLICY_LEDE = 0, 1, 2
+POLICY_AR, POLICY_STATIC, POLICY_LEDE, POLICY_THRESHOLD = 0, 1, 2, 3
 T_EMBED, T_LMHEAD, T_FINAL_NORM, T_ATTN_NORM, T_FFN_NORM, T_WQKV, T_WO, T_WGU, T_WDOWN = range(9)
 
 
@@ -43,7 +43,8 @@ class Policy(C.Structure):
     _fields_ = [("kind", C.c_int32), ("n_cand", C.c_int32), ("cand", C.c_int32 * MAX_CAND),
                 ("kmax", C.c_int32), ("static_l", C.c_int32), ("static_k", C.c_int32),
                 ("q_in", C.c_int32), ("q_hidden", C.c_int32), ("trace_T", C.c_int32),
-                ("topk", C.c_int32), ("q_params", C.c_void_p)]
+                ("topk", C.c_int32), ("q_params", C.c_void_p), ("fixed_k", C.c_int32),
+                ("conf_threshold", C.c_double)]
 
 
 class RoundLog(C.Structure):
@@ -172,7 +173,7 @@ def qnet(params: np.ndarray, hidden: int, s) -> np.ndarray:
 
 def make_policy(kind: int, cand=(), kmax: int = 0, static_l: int = 0, static_k: int = 0,
                 q_params: np.ndarray | None = None, q_hidden: int = 0, trace_T: int = 20,
-                topk: int = 5) -> Policy:
+                topk: int = 5, fixed_k: int = 0, conf_threshold: float = 0.0) -> Policy:
     P = Policy()
     P.kind = kind
     P.n_cand = len(cand)
@@ -180,6 +181,7 @@ def make_policy(kind: int, cand=(), kmax: int = 0, static_l: int = 0, static_k: 
         P.cand[i] = c
     P.kmax, P.static_l, P.static_k = kmax, static_l, static_k
     P.q_in, P.q_hidden, P.trace_T, P.topk = 3, q_hidden, trace_T, topk
+    P.fixed_k, P.conf_threshold = fixed_k, conf_threshold
     if q_params is not None:
         arr = np.ascontiguousarray(q_params, dtype=np.float32)
         P._keep = arr  # keep alive

@@ -557,6 +557,23 @@ static int q_decide(orc_sess* s, const orc_policy* P, const orc_stats* st, orc_r
   return a;
 }
 
+/* Draft & Verify-style rule (a §4.1 baseline): drafting goes on after a
+ * draft whose max-probability is at least the threshold.  Logged like a Q
+ * decision with values (threshold, pmax), so its margin is |pmax - tau|. */
+static int threshold_decide(const orc_policy* P, const orc_stats* st, orc_round_log* lg) {
+  int a = st->pmax >= P->conf_threshold ? 1 : 0;
+  if (lg->n_q < ORC_MAX_Q) {
+    int i = lg->n_q++;
+    lg->q_action[i] = a;
+    lg->q_val[i][0] = P->conf_threshold;
+    lg->q_val[i][1] = st->pmax;
+    lg->q_state[i][0] = st->conf_k;
+    lg->q_state[i][1] = st->entropy;
+    lg->q_state[i][2] = 0.0;
+  }
+  return a;
+}
+
 /* ------------------------------------------------------------ generation */
 
 static int check_policy(const orc_model* m, const orc_policy* P) {
@@ -567,7 +584,13 @@ static int check_policy(const orc_model* m, const orc_policy* P) {
     if (P->static_l < 1 || P->static_l > L || P->static_k < 1) return ORC_ERR_ARG;
     return ORC_OK;
   }
+  if (P->kind == ORC_POLICY_THRESHOLD) {
+    if (P->static_l < 1 || P->static_l > L) return ORC_ERR_ARG;
+    if (!(P->conf_threshold > 0.0 && P->conf_threshold <= 1.0)) return ORC_ERR_ARG;
+    return ORC_OK;
+  }
   if (P->kind != ORC_POLICY_LEDE) return ORC_ERR_ARG;
+  if (P->fixed_k < 0 || P->fixed_k > ORC_MAX_K - 1) return ORC_ERR_ARG;
   if (P->n_cand < 1 || P->n_cand > ORC_MAX_CAND || !P->q_params || P->q_in != 3 || P->q_hidden < 1 ||
       P->trace_T < 1)
     return ORC_ERR_ARG;
@@ -660,6 +683,8 @@ int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
   if (P->kind != ORC_POLICY_AR) {
     kcap = P->kmax < cap - 1 ? P->kmax : cap - 1;
     if (P->kind == ORC_POLICY_STATIC && P->static_k < kcap) kcap = P->static_k;
+    /* the ablation without adaptive drafting drafts a fixed length (Table 3) */
+    if (P->kind == ORC_POLICY_LEDE && P->fixed_k > 0 && P->fixed_k < kcap) kcap = P->fixed_k;
   }
   if (p + kcap + 1 > s->max_seq) return ORC_ERR_CAPACITY;
   lg->pos = p;
@@ -687,7 +712,13 @@ int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
       act = (j == n_c - 1) ? 1 : aq;
       if (act) {
         lstar = cj;
-        keep = aq;
+        /* whether d_1 is followed by more drafts */
+        if (P->kind == ORC_POLICY_THRESHOLD)
+          keep = threshold_decide(P, &st, lg);
+        else if (P->kind == ORC_POLICY_LEDE && P->fixed_k > 0)
+          keep = 1;
+        else
+          keep = aq;
         break;
       }
     }
@@ -703,7 +734,12 @@ int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
       drafts[k] = st.argmax;
       lg->draft_margin[k] = st.margin;
       ++k;
-      keep = P->kind == ORC_POLICY_LEDE ? q_decide(s, P, &st, lg) : 1;
+      if (P->kind == ORC_POLICY_THRESHOLD)
+        keep = threshold_decide(P, &st, lg);
+      else if (P->kind == ORC_POLICY_LEDE && P->fixed_k == 0)
+        keep = q_decide(s, P, &st, lg);
+      else
+        keep = 1;
     }
   }
   lg->k = k;

@@ -21,7 +21,7 @@
 #define ORC_TOPK_MAX 8
 
 enum { ORC_OK = 0, ORC_ERR_ARG = 1, ORC_ERR_CAPACITY = 2, ORC_ERR_STATE = 3, ORC_ERR_NOMEM = 4 };
-enum { ORC_POLICY_AR = 0, ORC_POLICY_STATIC = 1, ORC_POLICY_LEDE = 2 };
+enum { ORC_POLICY_AR = 0, ORC_POLICY_STATIC = 1, ORC_POLICY_LEDE = 2, ORC_POLICY_THRESHOLD = 3 };
 /* tensor selectors for orc_model_set / orc_model_get */
 enum {
   ORC_T_EMBED = 0, ORC_T_LMHEAD = 1, ORC_T_FINAL_NORM = 2, ORC_T_ATTN_NORM = 3, ORC_T_FFN_NORM = 4,
@@ -59,6 +59,8 @@ typedef struct {
   int32_t q_in, q_hidden;            /* q_in must be 3 */
   int32_t trace_T, topk;
   const float* q_params;             /* W1[h][in], b1[h], W2[2][h], b2[2] */
+  int32_t fixed_k;                   /* LEDE: 0 adaptive drafting; > 0 fixed draft length */
+  double conf_threshold;             /* THRESHOLD: drafting goes on while pmax >= this */
 } orc_policy;
 
 typedef struct {

@@ -34,6 +34,8 @@ struct RowSel {
 struct DevPolicy {
   int32_t kind, kmax, static_l, static_k, n_cand, q_hidden, trace_T, topk;
   int32_t cand[kMaxCand];
+  int32_t fixed_k;  // LEDE: fixed draft length (0: adaptive)
+  float tau;        // THRESHOLD: confidence threshold on a draft's max-probability
 };
 
 // Per-row statistics of an exit distribution (mirrors ssd_exit_stats).

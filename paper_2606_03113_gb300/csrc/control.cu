@@ -99,6 +99,7 @@ __global__ void k_round_begin(Dims D, Bufs B, cudaGraphConditionalHandle draft_i
   if (P.kind != SSD_POLICY_AR) {
     kcap = min(P.kmax, remaining - 1);
     if (P.kind == SSD_POLICY_STATIC) kcap = min(kcap, P.static_k);
+    if (P.kind == SSD_POLICY_LEDE && P.fixed_k > 0) kcap = min(kcap, P.fixed_k);
   }
   if (c->pos + kcap + 1 > D.max_seq) {
     atomicOr(&c->err, (int)kErrCapacity);
@@ -132,6 +133,9 @@ __global__ void k_round_begin(Dims D, Bufs B, cudaGraphConditionalHandle draft_i
 //         next walk segment (next_if).
 //  draft: record d_{k+1}; keep drafting while the action is exit and k < kcap.
 // Static policies exit at their only candidate and draft to their length.
+// Variants (Table 3, §4.1 baselines): LEDE with a fixed draft length uses the
+// Q-network only in the walk and drafts to the cap; THRESHOLD keeps drafting
+// while the draft's max-probability is >= tau (decision logged as (tau, pmax)).
 __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, int layer,
                          cudaGraphConditionalHandle next_if,
                          cudaGraphConditionalHandle draft_while) {
@@ -143,9 +147,11 @@ __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, in
   const DevPolicy& P = c->pol;
   const RowStats& st = B.stats[0];
   const bool lede = P.kind == SSD_POLICY_LEDE;
+  const bool thr = P.kind == SSD_POLICY_THRESHOLD;
+  const bool use_q = lede && (mode == kDecideWalk || P.fixed_k == 0);
   const int tid = threadIdx.x;
   float q0 = 0.f, q1 = 0.f;
-  if (lede) {
+  if (use_q) {
     if (tid == 0) {
       s_state[0] = st.conf_k;
       s_state[1] = st.entropy;
@@ -185,15 +191,17 @@ __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, in
   }
   if (tid != 0) return;
   ssd_round_trace& r = c->cur;
-  const int aq = lede ? (q1 > q0 ? 1 : 0) : 1;
-  if (lede && r.n_q < SSD_TRACE_MAXQ) {
+  const int aq = use_q ? (q1 > q0 ? 1 : 0) : 1;
+  // keep drafting after this decision?
+  const int go = thr ? (st.pmax >= P.tau ? 1 : 0) : ((lede && P.fixed_k > 0) ? 1 : aq);
+  if ((use_q || thr) && r.n_q < SSD_TRACE_MAXQ) {
     const int i = r.n_q++;
-    r.q_action[i] = aq;
-    r.q_val[i][0] = q0;
-    r.q_val[i][1] = q1;
-    r.q_state[i][0] = s_state[0];
-    r.q_state[i][1] = s_state[1];
-    r.q_state[i][2] = s_state[2];
+    r.q_action[i] = use_q ? aq : go;
+    r.q_val[i][0] = use_q ? q0 : P.tau;
+    r.q_val[i][1] = use_q ? q1 : st.pmax;
+    r.q_state[i][0] = use_q ? s_state[0] : st.conf_k;
+    r.q_state[i][1] = use_q ? s_state[1] : st.entropy;
+    r.q_state[i][2] = use_q ? s_state[2] : 0.f;
   }
   if (st.argmax < 0 || st.argmax >= D.V) atomicOr(&c->err, (int)kErrToken);
   if (mode == kDecideWalk) {
@@ -206,7 +214,7 @@ __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, in
       c->tok[1] = st.argmax;
       r.drafts[0] = st.argmax;
       r.draft_margin[0] = st.margin;
-      c->keep = (aq && 1 < c->kcap) ? 1 : 0;
+      c->keep = (go && 1 < c->kcap) ? 1 : 0;
       set_cond(next_if, 0u);
     } else {
       set_cond(next_if, 1u);
@@ -223,7 +231,7 @@ __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, in
     r.drafts[k] = st.argmax;
     r.draft_margin[k] = st.margin;
     c->k = k + 1;
-    c->keep = (aq && k + 1 < c->kcap) ? 1 : 0;
+    c->keep = (go && k + 1 < c->kcap) ? 1 : 0;
     set_cond(draft_while, (unsigned)c->keep);
   }
 }

@@ -136,7 +136,7 @@ struct ssd_ctx {
   bool have_policy = false;
   int kind = SSD_POLICY_AR;
   std::vector<int> cand;
-  int kmax = 0, static_l = 0, static_k = 0, q_hidden = 0, trace_T = 20, topk = 5;
+  int kmax = 0, static_l = 0, static_k = 0, q_hidden = 0, trace_T = 20, topk = 5, fixed_k = 0;
   // graphs
   cudaGraph_t round_g = nullptr, gen_g = nullptr;
   cudaGraphExec_t round_x = nullptr, gen_x = nullptr;
@@ -401,6 +401,7 @@ int kcap_for(const ssd_ctx* x, int budget) {
   if (x->kind == SSD_POLICY_AR) return 0;
   int k = std::min(x->kmax, budget - 1);
   if (x->kind == SSD_POLICY_STATIC) k = std::min(k, x->static_k);
+  if (x->kind == SSD_POLICY_LEDE && x->fixed_k > 0) k = std::min(k, x->fixed_k);
   return std::max(k, 0);
 }
 
@@ -525,7 +526,8 @@ ssd_status ssd_set_policy(ssd_ctx* x, const ssd_policy* p) {
   dp.topk = p->topk > 0 ? p->topk : 5;
   if (dp.trace_T > kTraceCap) return fail(x, SSD_ERR_INVALID_ARG, "trace_T must be in 1..64");
   if (dp.topk > kTopK) return fail(x, SSD_ERR_INVALID_ARG, "topk must be in 1..8");
-  if (p->kind != SSD_POLICY_AR && p->kind != SSD_POLICY_STATIC && p->kind != SSD_POLICY_LEDE)
+  if (p->kind != SSD_POLICY_AR && p->kind != SSD_POLICY_STATIC && p->kind != SSD_POLICY_LEDE &&
+      p->kind != SSD_POLICY_THRESHOLD)
     return fail(x, SSD_ERR_INVALID_ARG, "unknown policy kind");
   if (p->kind != SSD_POLICY_AR && (p->kmax < 1 || p->kmax > kMaxDraft))
     return fail(x, SSD_ERR_INVALID_ARG, "kmax must be in 1..16");
@@ -534,6 +536,14 @@ ssd_status ssd_set_policy(ssd_ctx* x, const ssd_policy* p) {
     if (p->static_l < 1 || p->static_l > L || p->static_k < 1)
       return fail(x, SSD_ERR_INVALID_ARG, "static_l must be in 1..n_layers and static_k >= 1");
   }
+  if (p->kind == SSD_POLICY_THRESHOLD) {
+    if (p->static_l < 1 || p->static_l > L)
+      return fail(x, SSD_ERR_INVALID_ARG, "static_l must be in 1..n_layers");
+    if (!(p->conf_threshold > 0.f && p->conf_threshold <= 1.f))
+      return fail(x, SSD_ERR_INVALID_ARG, "conf_threshold must be in (0, 1]");
+  }
+  if (p->kind == SSD_POLICY_LEDE && (p->fixed_k < 0 || p->fixed_k > kMaxDraft))
+    return fail(x, SSD_ERR_INVALID_ARG, "fixed_k must be in 0..16");
   if (p->kind == SSD_POLICY_LEDE) {
     if (p->n_cand < 1 || p->n_cand > kMaxCand || !p->cand_layers)
       return fail(x, SSD_ERR_INVALID_ARG, "n_cand must be in 1..16");
@@ -553,6 +563,8 @@ ssd_status ssd_set_policy(ssd_ctx* x, const ssd_policy* p) {
   dp.static_k = p->static_k;
   dp.n_cand = (int)cand.size();
   dp.q_hidden = p->kind == SSD_POLICY_LEDE ? p->qnet_hidden : 0;
+  dp.fixed_k = p->kind == SSD_POLICY_LEDE ? p->fixed_k : 0;
+  dp.tau = p->kind == SSD_POLICY_THRESHOLD ? p->conf_threshold : 0.f;
   CK(x, cudaMemcpyAsync(&x->B.ctl->pol, &dp, sizeof(dp), cudaMemcpyHostToDevice, x->stream));
   if (p->kind == SSD_POLICY_LEDE)
     CK(x, cudaMemcpyAsync(x->B.qparams, p->qnet_params, sizeof(float) * (6 * p->qnet_hidden + 2),
@@ -563,6 +575,7 @@ ssd_status ssd_set_policy(ssd_ctx* x, const ssd_policy* p) {
   x->kmax = p->kind == SSD_POLICY_AR ? 0 : p->kmax;
   x->static_l = p->static_l;
   x->static_k = p->static_k;
+  x->fixed_k = dp.fixed_k;
   x->q_hidden = dp.q_hidden;
   x->trace_T = dp.trace_T;
   x->topk = dp.topk;

@@ -19,7 +19,7 @@ SSD_ERR_STATE, SSD_ERR_DEVICE_FLAG, SSD_ERR_UNSUPPORTED = 4, 5, 6
 STATUS_NAMES = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_CUDA", 3: "SSD_ERR_CAPACITY",
                 4: "SSD_ERR_STATE", 5: "SSD_ERR_DEVICE_FLAG", 6: "SSD_ERR_UNSUPPORTED"}
 SSD_DTYPE_F32, SSD_DTYPE_BF16 = 0, 1
-SSD_POLICY_AR, SSD_POLICY_STATIC, SSD_POLICY_LEDE = 0, 1, 2
+SSD_POLICY_AR, SSD_POLICY_STATIC, SSD_POLICY_LEDE, SSD_POLICY_THRESHOLD = 0, 1, 2, 3
 TRACE_MAXK, TRACE_MAXQ, TRACE_MAXC = 16, 48, 16
 MAX_M = 17
 KERNELS_PER_LAYER = 5
@@ -44,7 +44,8 @@ class ssd_policy(C.Structure):
                 ("cand_layers", C.POINTER(C.c_int32)), ("kmax", C.c_int32),
                 ("static_l", C.c_int32), ("static_k", C.c_int32), ("qnet_in", C.c_int32),
                 ("qnet_hidden", C.c_int32), ("qnet_params", C.POINTER(C.c_float)),
-                ("trace_T", C.c_int32), ("topk", C.c_int32)]
+                ("trace_T", C.c_int32), ("topk", C.c_int32), ("fixed_k", C.c_int32),
+                ("conf_threshold", C.c_float)]
 
 
 class ssd_round_info(C.Structure):

@@ -28,53 +28,78 @@ def has_gpu() -> bool:
         return False
 
 
-def oracle_policy(kind: str, w, qp=None, l=0, k=0, kmax=None, cand=None):
+# Policy kinds: "ar", "static" (l, k), "lede" (cand; fixed_k > 0 drafts a
+# fixed length), "threshold" (l, tau).
+def oracle_policy(kind: str, w, qp=None, l=0, k=0, kmax=None, cand=None, fixed_k=0, tau=0.0):
     if kind == "ar":
         return oracle.make_policy(oracle.POLICY_AR)
     if kind == "static":
         return oracle.make_policy(oracle.POLICY_STATIC, kmax=kmax or k, static_l=l, static_k=k)
+    if kind == "threshold":
+        return oracle.make_policy(oracle.POLICY_THRESHOLD, kmax=kmax or w.kmax, static_l=l,
+                                  conf_threshold=tau)
     return oracle.make_policy(oracle.POLICY_LEDE, tuple(cand or w.candidates), kmax=kmax or w.kmax,
-                              q_params=qp, q_hidden=w.qnet_hidden)
+                              q_params=qp, q_hidden=w.qnet_hidden, fixed_k=fixed_k)
 
 
-def set_gpu_policy(eng, kind: str, w, qp=None, l=0, k=0, kmax=None, cand=None):
+def set_gpu_policy(eng, kind: str, w, qp=None, l=0, k=0, kmax=None, cand=None, fixed_k=0, tau=0.0):
     if kind == "ar":
         eng.set_ar()
     elif kind == "static":
         eng.set_static(l, k, kmax=kmax or k)
+    elif kind == "threshold":
+        eng.set_threshold(l, tau, kmax or w.kmax)
     else:
-        eng.set_lede(w, qp, kmax=kmax, cand=cand)
+        eng.set_lede(w, qp, kmax=kmax, cand=cand, fixed_k=fixed_k)
 
 
-def decisions(lg: dict, lede: bool) -> list:
+def decision_mode(kind: str, fixed_k: int = 0) -> str:
+    """"q": decisions in the walk and after every draft (LEDE, threshold);
+    "walk": in the walk only (LEDE with a fixed draft length); "none"."""
+    if kind == "threshold" or (kind == "lede" and not fixed_k):
+        return "q"
+    return "walk" if kind == "lede" else "none"
+
+
+def decisions(lg: dict, mode, thr: bool = False) -> list:
     """The round's decisions in the order they are taken: the walk's Q
-    decisions, d_1, then each further draft followed by the Q decision after
-    it, then the verification tokens g_0..g_k.  Each entry is
-    (kind, index, margin)."""
+    decisions, d_1, then each further draft followed by the decision after
+    it (mode "q"), then the verification tokens g_0..g_k.  Each entry is
+    (kind, index, margin).  Threshold decisions are logged as (tau, pmax);
+    their margin is |pmax - tau| / tau."""
+    if mode is True:
+        mode = "q"
+    elif mode is False:
+        mode = "none"
     out = []
-    nv = len(lg["visited"]) if lede else 0
-    for i in range(nv):
+
+    def margin(i):
         q0, q1 = lg["q_val"][i]
-        out.append(("q", i, abs(q1 - q0)))
+        return abs(q1 - q0) / q0 if thr else abs(q1 - q0)
+
+    nv = len(lg["visited"]) if mode != "none" else 0
+    if thr:
+        nv = 1 if lg["kcap"] > 0 else 0
+    for i in range(nv):
+        out.append(("q", i, margin(i)))
     k = lg["k"]
     for i in range(k):
         out.append(("d", i, lg["draft_margin"][i]))
-        if lede and i >= 1:
-            q0, q1 = lg["q_val"][nv + i - 1]
-            out.append(("q", nv + i - 1, abs(q1 - q0)))
+        if mode == "q" and i >= 1:
+            out.append(("q", nv + i - 1, margin(nv + i - 1)))
     for i in range(k + 1):
         out.append(("v", i, lg["verify_margin"][i]))
     return out
 
 
-def compare_round(g: dict, lg: dict, lede: bool, tol_tok: float, tol_q: float,
-                  q_val_tol: float):
+def compare_round(g: dict, lg: dict, lede, tol_tok: float, tol_q: float,
+                  q_val_tol: float, thr: bool = False):
     """Compares the GPU round g with the oracle round lg decision by decision
     up to the first decision the oracle takes with a margin at or below the
     tolerance.  Returns (compared, total, clear, max Q-value error)."""
     ctx = f"round at pos {lg['pos']}: gpu {g} oracle {lg}"
     assert g["pos"] == lg["pos"] and g["x"] == lg["x"] and g["kcap"] == lg["kcap"], ctx
-    ds = decisions(lg, lede)
+    ds = decisions(lg, lede, thr)
     n = 0
     q_err = 0.0
     for kind, i, margin in ds:
@@ -91,7 +116,7 @@ def compare_round(g: dict, lg: dict, lede: bool, tol_tok: float, tol_q: float,
             assert g["verify_tok"][i] == lg["verify_tok"][i], ("v", i, ctx)
         n += 1
     clear = n == len(ds)
-    walk_done = (not lede) or n >= len(lg["visited"])
+    walk_done = lede in (False, "none") or n >= len(lg["visited"])
     if walk_done and lg["kcap"] > 0:
         assert g["visited"] == lg["visited"] and g["lstar"] == lg["lstar"], ctx
     if clear:
@@ -108,13 +133,14 @@ def first_token_margin(om, ids) -> float:
 
 
 def generation_parity(eng, om, w, ids, kind: str, n_new: int, tol_tok: float, tol_q: float,
-                      q_val_tol: float, qp=None, l=0, k=0, kmax=None, cand=None) -> dict:
+                      q_val_tol: float, qp=None, l=0, k=0, kmax=None, cand=None, fixed_k=0,
+                      tau=0.0) -> dict:
     """Returns decision counts; asserts on every compared decision."""
-    P = oracle_policy(kind, w, qp, l, k, kmax, cand)
+    P = oracle_policy(kind, w, qp, l, k, kmax, cand, fixed_k, tau)
     s = om.session(eng.max_seq)
     ofirst = s.prefill(ids)
     otoks, logs = s.generate(P, n_new)
-    set_gpu_policy(eng, kind, w, qp, l, k, kmax, cand)
+    set_gpu_policy(eng, kind, w, qp, l, k, kmax, cand, fixed_k, tau)
     gfirst = eng.prefill(ids)
     seq = list(ids) + [ofirst]
     if gfirst != ofirst:
@@ -123,12 +149,13 @@ def generation_parity(eng, om, w, ids, kind: str, n_new: int, tol_tok: float, to
     compared = total = clear_rounds = 0
     q_err = 0.0
     done = 0
-    lede = kind == "lede"
+    mode = decision_mode(kind, fixed_k)
+    thr = kind == "threshold"
     for lg in logs:
         cap = n_new - done
         eng.step(cap)
         g = eng.traces(1)[0]
-        n, t, clear, qe = compare_round(g, lg, lede, tol_tok, tol_q, q_val_tol)
+        n, t, clear, qe = compare_round(g, lg, mode, tol_tok, tol_q, q_val_tol, thr)
         compared += n
         total += t
         clear_rounds += int(clear)

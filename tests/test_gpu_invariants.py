@@ -37,6 +37,15 @@ def test_ssd_equals_ar_bitwise_on_gpu():
             eng.prefill(ids)
             st, _, _ = eng.generate(w.gen_len)
             assert np.array_equal(ar, st), (name, l, k)
+        # the ablations of Table 3 and a confidence-threshold drafting rule
+        qp = synth.qnet_hidden_params(3, w.qnet_hidden, seed=2)
+        for setp in (lambda: eng.set_lede(w, qp, fixed_k=3),
+                     lambda: eng.set_lede(w, qp, cand=(w.candidates[0],)),
+                     lambda: eng.set_threshold(max(1, L // 2), 0.05, w.kmax)):
+            setp()
+            eng.prefill(ids)
+            va, _, _ = eng.generate(w.gen_len)
+            assert np.array_equal(ar, va), name
 
 
 def test_full_depth_exit_accepts_every_draft():

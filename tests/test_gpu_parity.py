@@ -215,3 +215,43 @@ def test_lede_always_exit_policy_drafts_to_cap():
                     assert t["visited"] == [w.candidates[0]] and t["k"] == t["kcap"]
                 else:
                     assert t["visited"] == list(w.candidates) and t["k"] == 1
+
+
+# --------------------------------------------- policy variants (Table 3, §4.1)
+
+
+def _median_exit_pmax(om, w, l):
+    """Median max-probability of the exit distribution at layer l over the
+    prompt (teacher forced): a threshold that splits the drafting decisions."""
+    s = om.session(w.max_seq)
+    ids = prompt(w)
+    h = s.forward(ids, 0, 0, l)
+    return float(np.median([om.exit_head(h[i])[1]["pmax"] for i in range(len(ids))]))
+
+
+@pytest.mark.parametrize("name", ["tiny", "7b", "8b"])
+@pytest.mark.parametrize("variant", ["no_dynamic_exit", "no_adaptive_drafting", "threshold"])
+def test_policy_variants_match_oracle(name, variant):
+    """The ablations of Table 3 (a single candidate exit layer; a fixed draft
+    length after the walk) and a Draft & Verify-style confidence threshold
+    run through the same graphs and kernels and match the oracle under the
+    same segment-and-resync protocol."""
+    w, dm, eng, om = setup(name)
+    tol_tok, tol_q, _, q_val_tol = TOL[w.shape.dtype]
+    qp = synth.qnet_hidden_params(3, w.qnet_hidden, seed=2)
+    L = w.shape.n_layers
+    if variant == "no_dynamic_exit":
+        kind, kw = "lede", dict(cand=(w.candidates[len(w.candidates) // 2],))
+    elif variant == "no_adaptive_drafting":
+        kind, kw = "lede", dict(fixed_k=min(4, w.kmax))
+    else:
+        l = max(1, L // 2)
+        kind, kw = "threshold", dict(l=l, tau=_median_exit_pmax(om, w, l))
+    r = generation_parity(eng, om, w, prompt(w), kind, w.gen_len, tol_tok, tol_q, q_val_tol,
+                          qp=qp, **kw)
+    print(name, variant, r)
+    need = 0.5 if w.shape.dtype == "f32" else 0.1
+    assert r["compared"] >= need * r["decisions"] and r["compared"] >= min(20, r["decisions"]), r
+    tr = eng.traces(4096)
+    if variant == "no_adaptive_drafting":
+        assert all(t["k"] == t["kcap"] for t in tr if t["kcap"] > 0)

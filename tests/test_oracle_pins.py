@@ -365,3 +365,107 @@ def test_error_paths():
         s.round(bad, 4)  # candidates must ascend
     with pytest.raises(oracle.OracleError):
         s.forward([9], 0, 0, 1)  # token out of vocabulary
+
+
+# ------------------------------------------------ policy variants (Table 3, §4.1)
+
+def _rounds(logs):
+    return [(lg["lstar"], lg["k"], lg["drafts"], lg["a"], lg["emitted"]) for lg in logs]
+
+
+@pytest.mark.parametrize("l,f", [(1, 2), (2, 3), (3, 4)])
+def test_fixed_length_single_candidate_is_static(tiny_setup, l, f):
+    """LEDE without dynamic exit and without adaptive drafting (one candidate,
+    fixed length) is exactly the static (l, f) policy, round for round, for
+    any Q-network: the only walk decision is a forced exit and the length is
+    not asked of the network."""
+    w, m, ids = tiny_setup
+    qp = synth.qnet_hidden_params(3, w.qnet_hidden, seed=3)
+    P = oracle.make_policy(oracle.POLICY_LEDE, (l,), kmax=w.kmax, q_params=qp,
+                           q_hidden=w.qnet_hidden, fixed_k=f)
+    S = oracle.make_policy(oracle.POLICY_STATIC, kmax=w.kmax, static_l=l, static_k=f)
+    _, a, la = generate(w, m, ids, P, 30)
+    _, b, lb = generate(w, m, ids, S, 30)
+    assert np.array_equal(a, b) and _rounds(la) == _rounds(lb)
+    # one Q decision per round (the walk), none after drafts
+    assert all(len(lg["q_action"]) == (1 if lg["kcap"] > 0 else 0) for lg in la)
+
+
+def test_fixed_length_keeps_the_walk(tiny_setup):
+    """Without adaptive drafting the walk still chooses l* by the Q-network
+    (always exit: the first candidate), and every speculative round drafts
+    min(fixed_k, cap) tokens."""
+    w, m, ids = tiny_setup
+    c = list(w.candidates)
+    for qc, qe, lstar in ((0.0, 1.0, c[0]), (1.0, 0.0, c[-1])):
+        P = oracle.make_policy(oracle.POLICY_LEDE, c, kmax=4, q_params=fixed_q(4, qc, qe),
+                               q_hidden=4, fixed_k=3)
+        out, logs = generate(w, m, ids, P, 25)[1:]
+        _, ar, _ = generate(w, m, ids, oracle.make_policy(oracle.POLICY_AR), 25)
+        assert np.array_equal(out, ar)
+        for lg in logs:
+            if lg["kcap"] > 0:
+                assert lg["lstar"] == lstar and lg["k"] == min(3, lg["kcap"]) == lg["kcap"]
+
+
+def test_single_candidate_adaptive_drafting(tiny_setup):
+    """Without dynamic exit (one candidate), an always-exit Q-network drafts
+    to the cap and a never-exit one drafts d_1 only: static (l, kmax) and
+    static (l, 1) round for round."""
+    w, m, ids = tiny_setup
+    for qc, qe, k in ((0.0, 1.0, w.kmax), (1.0, 0.0, 1)):
+        P = oracle.make_policy(oracle.POLICY_LEDE, (2,), kmax=w.kmax, q_params=fixed_q(4, qc, qe),
+                               q_hidden=4)
+        S = oracle.make_policy(oracle.POLICY_STATIC, kmax=w.kmax, static_l=2, static_k=k)
+        _, a, la = generate(w, m, ids, P, 30)
+        _, b, lb = generate(w, m, ids, S, 30)
+        assert np.array_equal(a, b) and _rounds(la) == _rounds(lb)
+
+
+def test_threshold_limits_and_rule(tiny_setup):
+    """Confidence-threshold drafting: a threshold no probability can miss
+    drafts to the cap (static (l, kmax)), one none can reach drafts d_1 only
+    (static (l, 1)); in between, each logged decision is pmax >= tau and
+    drafting stopped exactly at the first failed one or at the cap."""
+    w, m, ids = tiny_setup
+    pmax_seen = []
+    for tau, k in ((1e-12, w.kmax), (1.0, 1)):  # pmax < 1 for any spread distribution
+        P = oracle.make_policy(oracle.POLICY_THRESHOLD, kmax=w.kmax, static_l=2, conf_threshold=tau)
+        S = oracle.make_policy(oracle.POLICY_STATIC, kmax=w.kmax, static_l=2, static_k=k)
+        _, a, la = generate(w, m, ids, P, 30)
+        _, b, lb = generate(w, m, ids, S, 30)
+        assert np.array_equal(a, b) and _rounds(la) == _rounds(lb)
+        if tau < 1.0:
+            pmax_seen += [p for lg in la for _, p in lg["q_val"]]
+    # a threshold at the median observed draft confidence splits the decisions
+    tau = float(np.median(pmax_seen))
+    P = oracle.make_policy(oracle.POLICY_THRESHOLD, kmax=w.kmax, static_l=2, conf_threshold=tau)
+    out, logs = generate(w, m, ids, P, 40)[1:]
+    _, ar, _ = generate(w, m, ids, oracle.make_policy(oracle.POLICY_AR), 40)
+    assert np.array_equal(out, ar)
+    seen_both = set()
+    for lg in logs:
+        if lg["kcap"] == 0:
+            continue
+        acts = lg["q_action"]
+        assert len(acts) == lg["k"]  # one decision after each draft
+        for a, (t, p) in zip(acts, lg["q_val"]):
+            assert t == tau and a == (1 if p >= tau else 0)
+            seen_both.add(a)
+        stopped = [i for i, a in enumerate(acts) if a == 0]
+        assert lg["k"] == (stopped[0] + 1 if stopped else lg["kcap"])
+    assert seen_both == {0, 1}  # the threshold actually splits this run's decisions
+
+
+def test_variant_policies_rejected_when_malformed(tiny_setup):
+    w, m, ids = tiny_setup
+    s = m.session(w.max_seq)
+    s.prefill(ids)
+    bad = [oracle.make_policy(oracle.POLICY_THRESHOLD, kmax=4, static_l=2, conf_threshold=0.0),
+           oracle.make_policy(oracle.POLICY_THRESHOLD, kmax=4, static_l=2, conf_threshold=1.5),
+           oracle.make_policy(oracle.POLICY_THRESHOLD, kmax=4, static_l=0, conf_threshold=0.5),
+           oracle.make_policy(oracle.POLICY_LEDE, (1, 2), kmax=4, q_params=fixed_q(4, 0, 1),
+                              q_hidden=4, fixed_k=-1)]
+    for P in bad:
+        with pytest.raises(oracle.OracleError):
+            s.round(P, 10)
