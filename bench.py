@@ -285,6 +285,12 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="llama2-7b", choices=sorted(WORKLOADS))
     ap.add_argument("--policy", default="lede", choices=["lede", "ar", "static"])
+    ap.add_argument("--qnet", default="trained", choices=["trained", "seeded"],
+                    help="LEDE Q-network: trained offline by DQN on experience from this model "
+                         "(outside the timed region), or the seeded random network")
+    ap.add_argument("--train-prompts", type=int, default=4)
+    ap.add_argument("--train-gen", type=int, default=128)
+    ap.add_argument("--train-episodes", type=int, default=30000)
     ap.add_argument("--gen", type=int, default=0, help="new tokens per step (default: workload)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-compare", action="store_true", help="skip the AR / static lines")
@@ -330,13 +336,36 @@ def main():
     eng = Engine(model, w.max_seq, stream=stream)
     ids = synth.prompt_ids(w.prompt_len, w.shape.vocab)
 
-    def set_policy(kind, l=0, k=0):
+    seeded_qp = synth.qnet_hidden_params(3, w.qnet_hidden)
+    qnet_info = dict(kind="seeded")
+    qp = seeded_qp
+    if args.policy == "lede" and args.qnet == "trained" and not args.kernels_only:
+        # offline DQN (§3.2) on exit statistics of this model's own greedy
+        # continuations of prompts other than the benchmark's
+        from paper_2606_03113_gb300 import policy as PL
+        t0 = time.perf_counter()
+        prompts = [synth.prompt_ids(128, w.shape.vocab, seed=synth.SEED_PROMPT + 1 + i)
+                   for i in range(args.train_prompts)]
+        table = PL.collect_exit_table(eng, w.candidates, prompts, args.train_gen)
+        t1 = time.perf_counter()
+        qp, walk, tlog = PL.train_policy(table, w.qnet_hidden, episodes=args.train_episodes)
+        t2 = time.perf_counter()
+        qnet_info = dict(kind="trained (offline DQN)", positions=int(table.n),
+                         exit_agreement={int(c): round(float(a), 3)
+                                         for c, a in zip(w.candidates, table.agreement())},
+                         walk_return=round(walk["mean_return"], 4),
+                         walk_exit_layer=round(walk["exit_layer"], 2),
+                         hindsight_return=round(PL.oracle_walk_return(table), 4),
+                         updates=tlog.updates, collect_s=round(t1 - t0, 1),
+                         train_s=round(t2 - t1, 1))
+
+    def set_policy(kind, l=0, k=0, q=None):
         if kind == "ar":
             eng.set_ar()
         elif kind == "static":
             eng.set_static(l, k, kmax=w.kmax)
         else:
-            eng.set_lede(w, synth.qnet_hidden_params(3, w.qnet_hidden))
+            eng.set_lede(w, qp if q is None else q)
 
     L = w.shape.n_layers
     if args.kernels_only:
@@ -403,10 +432,13 @@ def main():
 
     compare = {}
     if not args.no_compare and args.policy == "lede":
-        for name, kind, lk in (("ar", "ar", (0, 0)), ("static_layerskip", "static", static_lk),
-                               ("static_l16_k4", "static", (L // 2, 4)),
-                               ("static_l24_k2", "static", (3 * L // 4, 2))):
-            set_policy(kind, *lk)
+        runs = [("ar", "ar", (0, 0), None), ("static_layerskip", "static", static_lk, None),
+                ("static_l16_k4", "static", (L // 2, 4), None),
+                ("static_l24_k2", "static", (3 * L // 4, 2), None)]
+        if qnet_info["kind"] != "seeded":
+            runs.append(("lede_seeded_qnet", "lede", (0, 0), seeded_qp))
+        for name, kind, lk, q in runs:
+            set_policy(kind, *lk, q=q)
             time_generate(eng, ids, n_new, barrier)
             r = time_generate(eng, ids, n_new, barrier)
             tr = r[2]
@@ -428,11 +460,12 @@ def main():
                 config=dict(workload=f"{w.name}-shaped decoder (random-init bf16), batch 1, "
                                      f"prompt {w.prompt_len}, {n_new} new tokens per step, "
                                      f"{args.policy} policy"
-                                     + (" (seeded Q-network)" if args.policy == "lede" else ""),
+                                     + ((" (" + qnet_info["kind"] + " Q-network)")
+                                        if args.policy == "lede" else ""),
                             l2="inputs larger than L2 (13.5 GB of weights streamed per pass)",
                             parallelism=f"replicas x{world}" if world > 1 else "single GPU"),
                 roofline=roofline, cpu_baseline=cpu, e2e=e2e, gpu_launches=launches,
-                clocks=clocks, policy_stats=policy_stats, compare=compare)
+                clocks=clocks, policy_stats=policy_stats, qnet=qnet_info, compare=compare)
     if rank == 0:
         print(json.dumps(line), flush=True)
     eng.close()

@@ -1,0 +1,365 @@
+"""Offline training of the LEDE exit policy (§3.1-§3.2, hyperparameters of
+§4.1), on experience read from the CUDA path.
+
+The hot path only evaluates the Q-network (k_decide); this module produces
+its weights, off the hot path, in plain numpy on the host:
+
+1. Experience (`collect_exit_table`): for sequences the model itself
+   generates greedily, every generated position is run teacher-forced
+   through `ssd_forward_exit` at each candidate exit layer and at the full
+   depth L.  A position's record holds, per candidate l, the state features
+   of §3.1.1 -- token confidence C_5 and entropy H of the exit distribution,
+   and the trace confidence C_trace of the full-model max-probabilities of
+   the previous T = 20 positions -- and whether the exit token x^l equals the
+   full-model token x^L (what acceptance of the draft needs).
+
+2. The MDP of §3.1 over one generation step: at candidate j the agent sees
+   s_j and picks continue (0) or exit (1); the last candidate forces exit.
+   Reward (§3.1.3): exit at l* gives 1 + (L - l*)/L if x^{l*} = x^L and
+   -2 + (L - l*)/L otherwise; continue gives -0.01.  An episode is the walk
+   of one generation step, started at a position drawn from the table.
+
+3. DQN (§3.2): a two-layer MLP Q(s) = W2 relu(W1 s + b1) + b2 with
+   factorised-Gaussian NoisyLinear layers (Fortunato et al., 2018; sigma_0 =
+   0.1) for exploration; n-step TD targets (n = 3, gamma = 0.99) from a
+   target network copied every 512 steps; Adam at 6.25e-5; 200 exploration
+   episodes before learning, then one update of 32 replayed transitions
+   every 4 agent steps.  The target's bootstrap value of a state where exit
+   is forced (the last candidate) is Q(s, exit).
+
+4. Deployment: the mean weights (noise off, §4.1) in the layout of
+   ssd_policy.qnet_params: W1[H][3], b1[H], W2[2][H], b2[2].
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass
+
+import numpy as np
+
+TRACE_T = 20
+GAMMA = 0.99
+N_STEP = 3
+LR = 6.25e-5
+SIGMA0 = 0.1
+EXPLORE_EPISODES = 200
+UPDATE_EVERY = 4
+BATCH = 32
+TARGET_EVERY = 512
+R_CONTINUE = -0.01
+
+
+# ------------------------------------------------------------- experience
+
+@dataclass
+class ExitTable:
+    """Per generated position t and candidate j: C_5, H at layer cands[j],
+    C_trace at t, and whether the exit token equals the full-model token."""
+    cands: tuple
+    n_layers: int
+    conf: np.ndarray     # [N, J]
+    ent: np.ndarray      # [N, J]
+    trace: np.ndarray    # [N]
+    correct: np.ndarray  # [N, J] bool
+    seqs: tuple = ()     # the token sequences (prompt + greedy continuation)
+
+    @property
+    def n(self) -> int:
+        return self.conf.shape[0]
+
+    def states(self) -> np.ndarray:
+        """[N, J, 3] state vectors (C_5, H, C_trace)."""
+        tr = np.broadcast_to(self.trace[:, None], self.conf.shape)
+        return np.stack([self.conf, self.ent, tr], axis=-1)
+
+    def agreement(self) -> np.ndarray:
+        """Fraction of positions whose exit token equals the full-model token,
+        per candidate layer."""
+        return self.correct.mean(axis=0)
+
+
+def _trace_conf(pmax_hist) -> float:
+    h = list(pmax_hist)[-TRACE_T:]
+    return -float(np.mean(np.log(h))) if h else 0.0
+
+
+def collect_exit_table(eng, cands, prompts, n_gen: int, chunk: int = 16) -> ExitTable:
+    """Experience from the CUDA path.  For each prompt: greedy generation of
+    n_gen tokens, then the generated positions teacher-forced in chunks at
+    every candidate layer (ascending) and at the full depth, which also
+    rewrites the chunk's KV rows for the next chunk."""
+    L = eng.shape.n_layers
+    cands = tuple(int(c) for c in cands)
+    rows_conf, rows_ent, rows_tr, rows_ok, seqs = [], [], [], [], []
+    for ids in prompts:
+        ids = [int(t) for t in ids]
+        eng.set_ar()
+        first = eng.prefill(ids)
+        gen, _, _ = eng.generate(n_gen)
+        seq = ids + [first] + [int(t) for t in gen]
+        seqs.append(seq)
+        eng.prefill(ids)  # reset the KV length; the prompt's trace seeds C_trace
+        _, _, trace = eng.read_state()
+        hist = [float(p) for p in trace]
+        p0 = len(ids)
+        for c0 in range(p0, p0 + n_gen, chunk):
+            toks = seq[c0:min(c0 + chunk, p0 + n_gen)]
+            per_l = {}
+            for l in cands + (L,):
+                _, st = eng.forward_exit(toks, c0, l, topk=5, logits=False)
+                per_l[l] = st
+            for i in range(len(toks)):
+                full = per_l[L][i]
+                rows_conf.append([per_l[l][i]["conf_k"] for l in cands])
+                rows_ent.append([per_l[l][i]["entropy"] for l in cands])
+                rows_tr.append(_trace_conf(hist))
+                rows_ok.append([per_l[l][i]["argmax"] == full["argmax"] for l in cands])
+                hist.append(max(float(full["pmax"]), 1e-30))
+    return ExitTable(cands, L, np.array(rows_conf, dtype=np.float64),
+                     np.array(rows_ent, dtype=np.float64), np.array(rows_tr, dtype=np.float64),
+                     np.array(rows_ok, dtype=bool), tuple(seqs))
+
+
+# ------------------------------------------------------------------ model
+
+def _f(x: np.ndarray) -> np.ndarray:
+    return np.sign(x) * np.sqrt(np.abs(x))
+
+
+class NoisyMLP:
+    """Q(s) = L2(relu(L1((s - mu) / sd))) over (continue, exit) with
+    factorised-Gaussian NoisyLinear layers: w = mu_w + sigma_w * (f(e_out)
+    f(e_in)^T), b = mu_b + sigma_b * f(e_out), f(x) = sign(x) sqrt|x|;
+    mu ~ U(+-1/sqrt(p)), sigma = sigma_0 / sqrt(p) (p = fan-in).  The state
+    is standardised with fixed statistics of the experience; export folds
+    them into the first layer, W1' = W1 / sd, b1' = b1 - W1' mu, so the
+    deployed network reads the raw state (C_5, H, C_trace).  Plain numpy:
+    the network is tiny and an update is a handful of small matrix products.
+    Adam with PyTorch's default moments (0.9, 0.999, 1e-8)."""
+
+    def __init__(self, hidden: int, sigma0: float, rng: np.random.Generator, mu, sd):
+        self.rng = rng
+        self.mu, self.sd = np.asarray(mu, np.float64), np.asarray(sd, np.float64)
+        b1, b2 = 1.0 / math.sqrt(3), 1.0 / math.sqrt(hidden)
+        self.p = {
+            "w1": rng.uniform(-b1, b1, (hidden, 3)), "b1": rng.uniform(-b1, b1, hidden),
+            "sw1": np.full((hidden, 3), sigma0 * b1), "sb1": np.full(hidden, sigma0 * b1),
+            "w2": rng.uniform(-b2, b2, (2, hidden)), "b2": rng.uniform(-b2, b2, 2),
+            "sw2": np.full((2, hidden), sigma0 * b2), "sb2": np.full(2, sigma0 * b2),
+        }
+        self.m = {k: np.zeros_like(v) for k, v in self.p.items()}
+        self.v = {k: np.zeros_like(v) for k, v in self.p.items()}
+        self.t = 0
+        self.reset_noise()
+
+    def reset_noise(self):
+        H = self.p["b1"].size
+        self.ei1, self.eo1 = _f(self.rng.normal(size=3)), _f(self.rng.normal(size=H))
+        self.ei2, self.eo2 = _f(self.rng.normal(size=H)), _f(self.rng.normal(size=2))
+
+    def _weights(self, noisy: bool):
+        p = self.p
+        if not noisy:
+            return p["w1"], p["b1"], p["w2"], p["b2"]
+        return (p["w1"] + p["sw1"] * np.outer(self.eo1, self.ei1), p["b1"] + p["sb1"] * self.eo1,
+                p["w2"] + p["sw2"] * np.outer(self.eo2, self.ei2), p["b2"] + p["sb2"] * self.eo2)
+
+    def q(self, s: np.ndarray, noisy: bool = True) -> np.ndarray:
+        w1, b1, w2, b2 = self._weights(noisy)
+        x = (s - self.mu) / self.sd
+        return np.maximum(x @ w1.T + b1, 0.0) @ w2.T + b2
+
+    def sgd_step(self, s, a, y, lr: float):
+        """One Adam step on mean((Q(s)[a] - y)^2) with the current noise."""
+        w1, b1, w2, b2 = self._weights(True)
+        x = (s - self.mu) / self.sd
+        z1 = x @ w1.T + b1
+        h = np.maximum(z1, 0.0)
+        q = h @ w2.T + b2
+        B = s.shape[0]
+        dq = np.zeros_like(q)
+        dq[np.arange(B), a] = 2.0 * (q[np.arange(B), a] - y) / B
+        dw2 = dq.T @ h
+        db2 = dq.sum(axis=0)
+        dz1 = (dq @ w2) * (z1 > 0)
+        dw1 = dz1.T @ x
+        db1 = dz1.sum(axis=0)
+        g = {"w1": dw1, "b1": db1, "sw1": dw1 * np.outer(self.eo1, self.ei1), "sb1": db1 * self.eo1,
+             "w2": dw2, "b2": db2, "sw2": dw2 * np.outer(self.eo2, self.ei2), "sb2": db2 * self.eo2}
+        self.t += 1
+        c1, c2 = 1.0 - 0.9 ** self.t, 1.0 - 0.999 ** self.t
+        for k, gk in g.items():
+            self.m[k] = 0.9 * self.m[k] + 0.1 * gk
+            self.v[k] = 0.999 * self.v[k] + 0.001 * gk * gk
+            self.p[k] -= lr * (self.m[k] / c1) / (np.sqrt(self.v[k] / c2) + 1e-8)
+
+    def copy_means_from(self, other: "NoisyMLP"):
+        for k in ("w1", "b1", "w2", "b2"):
+            self.p[k] = other.p[k].copy()
+
+    def export(self) -> np.ndarray:
+        """Mean weights as ssd_policy.qnet_params: W1[H][3], b1[H], W2[2][H], b2[2]."""
+        w1 = self.p["w1"] / self.sd[None, :]
+        b1 = self.p["b1"] - w1 @ self.mu
+        parts = [w1, b1, self.p["w2"], self.p["b2"]]
+        return np.concatenate([x.reshape(-1) for x in parts]).astype(np.float32)
+
+
+# -------------------------------------------------------------- training
+
+def walk_reward(table: ExitTable, t: int, j: int) -> float:
+    L = table.n_layers
+    l = table.cands[j]
+    return (1.0 if table.correct[t, j] else -2.0) + (L - l) / L
+
+
+@dataclass
+class TrainLog:
+    episodes: int
+    updates: int
+    mean_return: list       # mean undiscounted return per block of episodes
+    exit_layer: list        # mean chosen exit layer per block
+    agreement: list         # fraction of exits whose token was correct per block
+
+
+def train_dqn(table: ExitTable, hidden: int, episodes: int, seed: int = 0, parallel: int = 64,
+              block: int = 2000) -> tuple[np.ndarray, TrainLog]:
+    """DQN on the walk MDP of `table` (§3.2) with the §4.1 schedule; returns
+    the deployed weights and the learning curve.  Walks run `parallel` at a
+    time under one noise sample; the schedule is kept per agent step (one
+    update of BATCH transitions per UPDATE_EVERY steps, with fresh noise;
+    target copy every TARGET_EVERY steps; learning after EXPLORE_EPISODES
+    episodes)."""
+    rng = np.random.default_rng(seed)
+    S = table.states()  # [N, J, 3]
+    flat = S.reshape(-1, 3)
+    mu, sd = flat.mean(axis=0), flat.std(axis=0) + 1e-6
+    online = NoisyMLP(hidden, SIGMA0, rng, mu, sd)
+    target = NoisyMLP(hidden, SIGMA0, rng, mu, sd)
+    target.copy_means_from(online)
+    J = len(table.cands)
+    cand = np.array(table.cands)
+    R_exit = np.where(table.correct, 1.0, -2.0) + (table.n_layers - cand[None, :]) / table.n_layers
+    cap = 200_000
+    bs = np.zeros((cap, 3))
+    ba = np.zeros(cap, dtype=np.int64)
+    bG = np.zeros(cap)
+    bsb = np.zeros((cap, 3))
+    bdisc = np.zeros(cap)
+    bforced = np.zeros(cap, dtype=bool)
+    n_buf = w_buf = 0
+    steps = updates = done_eps = next_target = 0
+    curve_ret, curve_l, curve_ok = [], [], []
+    acc = [0.0, 0.0, 0.0, 0]
+
+    def update():
+        idx = rng.integers(0, n_buf, BATCH)
+        qb = target.q(bsb[idx], noisy=False)
+        vb = np.where(bforced[idx], qb[:, 1], qb.max(axis=1))
+        y = bG[idx] + bdisc[idx] * vb
+        online.reset_noise()
+        online.sgd_step(bs[idx], ba[idx], y, LR)
+
+    while done_eps < episodes:
+        P = min(parallel, episodes - done_eps)
+        ts = rng.integers(0, table.n, P)
+        online.reset_noise()
+        q = online.q(S[ts])  # [P, J, 2]
+        act = q[..., 1] > q[..., 0]  # ties continue
+        act[:, J - 1] = True
+        jx = act.argmax(axis=1)  # exit index of each walk
+        n_steps = int((jx + 1).sum())
+        # transitions with n-step returns (exit terminal; forced exit at the last candidate)
+        e_idx = np.repeat(np.arange(P), jx + 1)
+        i_idx = np.concatenate([np.arange(j + 1) for j in jx])
+        t_idx = ts[e_idx]
+        je = jx[e_idx]
+        rexit = R_exit[ts, jx]  # [P]
+
+        def rew(off):
+            k = i_idx + off
+            r = np.where(k < je, R_CONTINUE, rexit[e_idx])
+            return np.where(k <= je, r, 0.0)
+
+        G = sum((GAMMA ** k) * rew(k) for k in range(N_STEP))
+        boot = i_idx + N_STEP <= je
+        jb = np.where(boot, i_idx + N_STEP, i_idx)
+        n_new = len(e_idx)
+        pos = (w_buf + np.arange(n_new)) % cap
+        bs[pos] = S[t_idx, i_idx]
+        ba[pos] = (i_idx == je).astype(np.int64)
+        bG[pos] = G
+        bsb[pos] = S[t_idx, jb]
+        bdisc[pos] = np.where(boot, GAMMA ** N_STEP, 0.0)
+        bforced[pos] = boot & (jb == J - 1)
+        w_buf = int((w_buf + n_new) % cap)
+        n_buf = min(n_buf + n_new, cap)
+        acc[0] += float(R_CONTINUE * jx.sum() + rexit.sum())
+        acc[1] += float(cand[jx].sum())
+        acc[2] += float(table.correct[ts, jx].sum())
+        acc[3] += P
+        prev = steps
+        steps += n_steps
+        done_eps += P
+        if done_eps > EXPLORE_EPISODES and n_buf >= BATCH:
+            for _ in range(steps // UPDATE_EVERY - prev // UPDATE_EVERY):
+                update()
+                updates += 1
+        while next_target + TARGET_EVERY <= steps:
+            next_target += TARGET_EVERY
+            target.copy_means_from(online)
+        if acc[3] >= block:
+            curve_ret.append(acc[0] / acc[3])
+            curve_l.append(acc[1] / acc[3])
+            curve_ok.append(acc[2] / acc[3])
+            acc = [0.0, 0.0, 0.0, 0]
+    return online.export(), TrainLog(episodes, updates, curve_ret, curve_l, curve_ok)
+
+
+def greedy_walk_stats(params: np.ndarray, hidden: int, table: ExitTable) -> dict:
+    """The deployed (noise-free) policy's walk on every position of the
+    table: mean return, mean exit layer, fraction of correct exits."""
+    W1 = params[:3 * hidden].reshape(hidden, 3).astype(np.float64)
+    b1 = params[3 * hidden:4 * hidden].astype(np.float64)
+    W2 = params[4 * hidden:6 * hidden].reshape(2, hidden).astype(np.float64)
+    b2 = params[6 * hidden:6 * hidden + 2].astype(np.float64)
+    S = table.states()
+    J = len(table.cands)
+    rets, ls, oks = [], [], []
+    for t in range(table.n):
+        ret = 0.0
+        for j in range(J):
+            q = W2 @ np.maximum(W1 @ S[t, j] + b1, 0.0) + b2
+            if j == J - 1 or q[1] > q[0]:
+                ret += walk_reward(table, t, j)
+                ls.append(table.cands[j])
+                oks.append(bool(table.correct[t, j]))
+                break
+            ret += R_CONTINUE
+        rets.append(ret)
+    return dict(mean_return=float(np.mean(rets)), exit_layer=float(np.mean(ls)),
+                correct=float(np.mean(oks)))
+
+
+def train_policy(table: ExitTable, hidden: int, episodes: int = 30000, seeds=(0, 1, 2)):
+    """DQN runs from several seeds (a run can settle on exiting at the first
+    candidate when its initial network prefers exit there); the deployed
+    policy is the one whose greedy walk earns the highest mean return on the
+    experience.  Returns (params, walk stats, log of the chosen run)."""
+    best = None
+    for seed in seeds:
+        params, log = train_dqn(table, hidden, episodes, seed=seed)
+        st = greedy_walk_stats(params, hidden, table)
+        if best is None or st["mean_return"] > best[1]["mean_return"]:
+            best = (params, st, log)
+    return best
+
+
+def oracle_walk_return(table: ExitTable) -> float:
+    """Mean return of the best exit in hindsight at every position (an upper
+    bound for any policy on the table)."""
+    J = len(table.cands)
+    cand = np.array(table.cands)
+    R = np.where(table.correct, 1.0, -2.0) + (table.n_layers - cand[None, :]) / table.n_layers
+    R = R + R_CONTINUE * np.arange(J)[None, :]
+    return float(R.max(axis=1).mean())

@@ -255,3 +255,39 @@ def test_policy_variants_match_oracle(name, variant):
     tr = eng.traces(4096)
     if variant == "no_adaptive_drafting":
         assert all(t["k"] == t["kcap"] for t in tr if t["kcap"] > 0)
+
+
+# ------------------------------------------- experience for the offline DQN
+
+
+def test_exit_table_collection_matches_oracle():
+    """Experience for the offline DQN (§3.2) read through the C ABI: the
+    greedy continuation is the oracle's where its decisions are clear, and
+    each sampled position's exit statistics (C_5, H, exit token) at every
+    candidate equal the oracle's teacher-forced exit head within the logits
+    tolerance; C_trace follows the full-model max-probabilities."""
+    from paper_2606_03113_gb300 import policy as P
+    w, dm, eng, om = setup("7b")
+    ids = prompt(w, 40)
+    n_gen = 24
+    tab = P.collect_exit_table(eng, w.candidates, [ids], n_gen)
+    J = len(w.candidates)
+    assert tab.conf.shape == (n_gen, J) and tab.correct.shape == (n_gen, J)
+    # the same positions through the oracle, teacher-forced on the GPU's own
+    # greedy continuation
+    seq = tab.seqs[0]
+    assert seq[:len(ids)] == list(ids) and len(seq) == len(ids) + n_gen + 1
+    L = w.shape.n_layers
+    hL = om.session(w.max_seq).forward(seq[:len(ids) + n_gen], 0, 0, L)
+    for j, c in enumerate(w.candidates):
+        h = om.session(w.max_seq).forward(seq[:len(ids) + n_gen], 0, 0, c)
+        for t in range(0, n_gen, 5):
+            _, sr = om.exit_head(h[len(ids) + t])
+            _, sf = om.exit_head(hL[len(ids) + t])
+            assert abs(tab.conf[t, j] - sr["conf_k"]) <= 2e-2 * max(1.0, sr["conf_k"])
+            assert abs(tab.ent[t, j] - sr["entropy"]) <= 2e-2 * max(1.0, sr["entropy"])
+            if sr["margin"] > 5e-2 and sf["margin"] > 5e-2:
+                assert tab.correct[t, j] == (sr["argmax"] == sf["argmax"]), (c, t)
+    # C_trace at the first generated position: the prompt's last 20 full-model rows
+    tr0 = -np.mean([np.log(om.exit_head(hL[r])[1]["pmax"]) for r in range(len(ids) - 20, len(ids))])
+    assert abs(tab.trace[0] - tr0) <= 2e-2 * max(1.0, tr0)
