@@ -204,6 +204,23 @@ def run_reference(args, w, rank: int, world: int):
     print(json.dumps(line), flush=True)
 
 
+# ------------------------------------------------------------- replicas
+
+def aggregate_replicas(local_ms: float, local_tokens: float, device: str = "cpu") -> tuple:
+    """Whole-job timing of N independent replicas (one sequence per rank, no
+    data-path collective): the slowest rank's time and the tokens of all
+    ranks.  A no-op without an initialised process group of size > 1."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1):
+        return float(local_ms), float(local_tokens)
+    mx = torch.tensor([float(local_ms)], dtype=torch.float64, device=device)
+    tot = torch.tensor([float(local_tokens)], dtype=torch.float64, device=device)
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    dist.all_reduce(tot, op=dist.ReduceOp.SUM)
+    return float(mx[0]), float(tot[0])
+
+
 # ------------------------------------------------------------------ GPU arm
 
 def time_generate(eng, ids, n_new, dist_barrier) -> tuple:
@@ -388,14 +405,7 @@ def main():
     ms = [r[0] for r in results]
     toks = [r[1] for r in results]
     local_ms = sum(ms)
-    if world > 1:
-        t = torch.tensor([local_ms, float(sum(toks))], device=f"cuda:{local}")
-        mx = t.clone()
-        dist.all_reduce(mx[:1], op=dist.ReduceOp.MAX)
-        dist.all_reduce(t[1:], op=dist.ReduceOp.SUM)
-        total_ms, total_tok = float(mx[0]), float(t[1])
-    else:
-        total_ms, total_tok = local_ms, float(sum(toks))
+    total_ms, total_tok = aggregate_replicas(local_ms, float(sum(toks)), f"cuda:{local}")
     value = total_tok / (total_ms / 1e3)
     traces = results[-1][2]
     bytes_step = sum(round_bytes(w, tr) for tr in traces)
