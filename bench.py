@@ -46,18 +46,22 @@ def measured_peaks() -> dict:
     return dict(hbm_gbs=6800.0, src="fallback")
 
 
-# DRAM traffic of the dominant kernel from the committed ncu summary: valid
+# DRAM traffic of the dominant kernel from the committed ncu summaries: valid
 # only while the kernel's sources are the ones that were captured.
-TRAFFIC_PROFILE = os.path.join(REPO, "profiles", "k_tile_gate_up_llama2-7b.md")
+TRAFFIC_PROFILES = {"k_gate_up": "k_tile_gate_up_llama2-7b.md",
+                    "k_chain(o+gate_up+down+next_qkv)": "k_chain_llama2-7b.md"}
 TRAFFIC_SOURCES = ("tile.cu", "tc.cuh", "pipe.cuh", "headpart.cuh")
 
 
-def measured_traffic() -> int | None:
-    """DRAM read + write bytes per single-row gate/up launch (Llama-2-7B
-    shape) from one ncu capture, or None when the summary is missing or the
-    kernel sources no longer hash to the captured value."""
+def measured_traffic(kernel: str) -> int | None:
+    """DRAM read + write bytes per single-row launch of `kernel` on the
+    Llama-2-7B shape from one ncu capture, or None when there is no summary
+    or the kernel sources no longer hash to the captured value."""
+    name = TRAFFIC_PROFILES.get(kernel)
+    if name is None:
+        return None
     try:
-        text = open(TRAFFIC_PROFILE).read()
+        text = open(os.path.join(REPO, "profiles", name)).read()
         h = hashlib.sha256()
         for f in TRAFFIC_SOURCES:
             with open(os.path.join(REPO, "paper_2606_03113_gb300", "csrc", f), "rb") as fh:
@@ -95,7 +99,7 @@ def round_bytes(w, tr: dict) -> float:
 
 def kernels_in_round(w, tr: dict) -> int:
     from paper_2606_03113_gb300.runtime import kernels_per_round
-    return kernels_per_round(tr, w.shape.n_layers, 0)
+    return kernels_per_round(tr, w.shape.n_layers, 0, bf16=w.shape.dtype == "bf16")
 
 
 # ------------------------------------------------------------------ clocks
@@ -239,7 +243,7 @@ def time_generate(eng, ids, n_new, dist_barrier) -> tuple:
 
 
 KERNEL_NAMES = {0: "k_qkv", 1: "k_attn", 2: "k_resid(wo)", 3: "k_gate_up",
-                4: "k_resid(w_down)", 5: "k_head"}
+                4: "k_resid(w_down)", 5: "k_head", 6: "k_chain(o+gate_up+down+next_qkv)"}
 
 
 def kernel_roofline(eng, w, peak: float, pos0: int, iters: int = 5, graphs: bool = True) -> dict:
@@ -257,9 +261,15 @@ def kernel_roofline(eng, w, peak: float, pos0: int, iters: int = 5, graphs: bool
     byts = {0: s.qkv_rows * s.d_model * elt, 1: s.kv_bytes_per_pos_layer() * (pos0 + 1),
             2: s.d_model * qd * elt, 3: 2 * s.ffn_dim * s.d_model * elt,
             4: s.d_model * s.ffn_dim * elt, 5: s.vocab * s.d_model * elt}
+    kerns = (0, 1, 2, 3, 4, 5)
+    if s.dtype == "bf16":
+        # the chained launch the layer passes use: O, gate/up, down of layer
+        # l and the QKV of layer l + 1 (the last layer has no QKV phase)
+        byts[6] = byts[2] + byts[3] + byts[4] + byts[0] * (L - 1) / L
+        kerns = kerns + (6,)
     out = {}
     st = eng.stream
-    for kern in (0, 1, 2, 3, 4, 5):
+    for kern in kerns:
         layers = [0] * 8 if kern == 5 else list(range(L))
 
         def run():
@@ -430,8 +440,12 @@ def main():
                note="ssd_prefill (host prompt) + ssd_generate (host tokens), wall clock")
 
     roof = kernel_roofline(eng, w, peak, pos0=w.prompt_len + n_new // 2)
-    dom = max(roof.items(), key=lambda kv: kv[1]["us"] * kv[1]["launches_per_forward"])
-    traffic = measured_traffic() if (w.name == "llama2-7b" and dom[0] == "k_gate_up") else None
+    # the dominant kernel among those a forward pass launches (bf16: the
+    # chained launch replaces the per-matrix ones)
+    launched = {k: v for k, v in roof.items()
+                if KERNEL_NAMES[6] not in roof or k in (KERNEL_NAMES[6], "k_attn", "k_head")}
+    dom = max(launched.items(), key=lambda kv: kv[1]["us"] * kv[1]["launches_per_forward"])
+    traffic = measured_traffic(dom[0]) if w.name == "llama2-7b" else None
     roofline = dict(bound="hbm", achieved=dom[1]["gbs"], peak=peak, unit="GB/s",
                     frac=dom[1]["gbs"] / peak, traffic=traffic,
                     kernel=f"{dom[0]} single-row ({dom[1]['bytes'] / 1e6:.1f} MB per launch)",

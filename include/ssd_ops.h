@@ -62,7 +62,9 @@ ssd_status ssd_op_gemv(ssd_ctx* ctx, int32_t which, int32_t layer, int32_t M, co
  * own buffers: kernel = 0 QKV (+RoPE, KV append), 1 attention (split-K with
  * the split merge in the same kernel), 2 O projection (+residual), 3 gate/up (+RMSNorm, SwiGLU),
  * 4 down projection (+residual), 5 exit head (final RMSNorm, LM head,
- * statistics; layer ignored).  It overwrites the activations and the KV rows
+ * statistics; layer ignored), 6 (bf16) the chained launch the layer passes
+ * use: O projection, gate/up and down of `layer` and the QKV of layer + 1
+ * (when there is one) as the phases of one persistent kernel.  It overwrites the activations and the KV rows
  * at those positions: for timing and profiling, not inside a generation.
  * Needs pos0 + M <= max_seq.  Enqueued on `stream` (NULL = the context's). */
 ssd_status ssd_op_layer(ssd_ctx* ctx, int32_t kernel, int32_t layer, int32_t M, int32_t pos0,

@@ -164,6 +164,7 @@ struct Bufs {
   float* attn_part;  // [kMaxM][Hq][nsplit][hd] unnormalised partial outputs
   float* attn_ml;    // [kMaxM][Hq][nsplit][2] partial (max, sum)
   uint32_t* attn_counter;  // [Hkv][kMaxM] split tickets of the attention merge
+  uint32_t* chain_bar;     // [2] grid-wide phase arrivals / blocks done of the chain kernel
   float* attn_out;   // [kMaxM][qd]
   float* act;        // [kMaxM][F]
   float* logits;     // [kMaxM][V] (written only when requested)

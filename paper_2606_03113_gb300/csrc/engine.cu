@@ -81,6 +81,7 @@ size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
   b.attn_part = cv.take<float>(sizeof(float) * kMaxM * d.Hq * (size_t)d.nsplit * d.hd);
   b.attn_ml = cv.take<float>(sizeof(float) * kMaxM * d.Hq * (size_t)d.nsplit * 2);
   b.attn_counter = cv.take<uint32_t>(sizeof(uint32_t) * (size_t)d.Hkv * kMaxM);
+  b.chain_bar = cv.take<uint32_t>(sizeof(uint32_t) * 2);
   b.attn_out = cv.take<float>(sizeof(float) * kMaxM * d.qd);
   b.act = cv.take<float>(sizeof(float) * kMaxM * d.F);
   b.logits = cv.take<float>(sizeof(float) * kMaxM * (size_t)d.V);
@@ -229,6 +230,19 @@ const CUtensorMap* lm_map(const ssd_ctx* x) {
 // mrows: the most rows the launches will see (1: the single-row kernels).
 cudaError_t enqueue_layers(ssd_ctx* x, int l_from, int l_to, RowSel sel, int mrows,
                            cudaStream_t st) {
+  if (x->cfg.dtype == SSD_DTYPE_BF16 && g_chain_enabled && l_to > l_from) {
+    // QKV of the first layer, then per layer: attention, and O + gate/up +
+    // down + the next layer's QKV as one persistent launch
+    GK(launch_layer_part(x->D, x->B, x->cfg.dtype, x->layers[l_from], tile_maps(x), l_from, 0, sel,
+                         mrows, st));
+    for (int l = l_from; l < l_to; ++l) {
+      GK(launch_layer_part(x->D, x->B, x->cfg.dtype, x->layers[l], tile_maps(x), l, 1, sel, mrows,
+                           st));
+      GK(launch_tile_chain(x->D, x->B, *tile_maps(x), x->layers[l],
+                           l + 1 < l_to ? &x->layers[l + 1] : nullptr, l, sel, mrows, st));
+    }
+    return cudaSuccess;
+  }
   for (int l = l_from; l < l_to; ++l)
     GK(launch_layer(x->D, x->B, x->cfg.dtype, x->layers[l], tile_maps(x), l, sel, mrows, st));
   return cudaSuccess;
@@ -443,6 +457,7 @@ ssd_status ssd_init_model(const ssd_model_cfg* cfg, const ssd_weights* w, void* 
   if (e0 == cudaSuccess && cfg->dtype == SSD_DTYPE_BF16) e0 = prepare_tile_kernels();
   if (e0 != cudaSuccess) return cuda_fail(nullptr, "ssd_init_model device query", e0);
   if (const char* v = getenv("SSD_NO_PDL")) g_pdl_enabled = !(v[0] == '1');
+  if (const char* v = getenv("SSD_NO_CHAIN")) g_chain_enabled = !(v[0] == '1');
   ssd_ctx* x = new ssd_ctx();
   x->cfg = *cfg;
   layout(*cfg, static_cast<char*>(workspace), &x->D, &x->B);
@@ -503,6 +518,7 @@ ssd_status ssd_init_model(const ssd_model_cfg* cfg, const ssd_weights* w, void* 
   if (e == cudaSuccess) e = cudaMemsetAsync(x->B.ss_counter, 0, sizeof(uint32_t) * 2, x->stream);
   if (e == cudaSuccess)
     e = cudaMemsetAsync(x->B.attn_counter, 0, sizeof(uint32_t) * (size_t)x->D.Hkv * kMaxM, x->stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(x->B.chain_bar, 0, sizeof(uint32_t) * 2, x->stream);
   if (e == cudaSuccess)
     e = cudaMemsetAsync(x->B.tile_counter, 0, sizeof(uint32_t) * (size_t)x->D.max_tiles, x->stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(x->stream);
@@ -870,12 +886,18 @@ ssd_status ssd_op_layer(ssd_ctx* x, int32_t kernel, int32_t layer, int32_t M, in
   if (!x) return fail(nullptr, SSD_ERR_INVALID_ARG, "ctx is NULL");
   if (M < 1 || M > kMaxM || pos0 < 0 || pos0 + M > x->cfg.max_seq)
     return fail(x, SSD_ERR_INVALID_ARG, "M must be in 1..17 with pos0 + M <= max_seq");
-  if (kernel < 0 || kernel > 5 || (kernel < 5 && (layer < 0 || layer >= x->cfg.n_layers)))
-    return fail(x, SSD_ERR_INVALID_ARG, "kernel must be 0..5 and layer in range");
+  if (kernel < 0 || kernel > 6 || (kernel != 5 && (layer < 0 || layer >= x->cfg.n_layers)))
+    return fail(x, SSD_ERR_INVALID_ARG, "kernel must be 0..6 and layer in range");
+  if (kernel == 6 && x->cfg.dtype != SSD_DTYPE_BF16)
+    return fail(x, SSD_ERR_INVALID_ARG, "the chained kernel is a bf16 kernel");
   cudaStream_t st = stream ? static_cast<cudaStream_t>(stream) : x->stream;
   const RowSel sel = rows_explicit(pos0, M, x->B.pre_tok);
   if (kernel == 5)
     CK(x, enqueue_head(x, sel, M, x->topk, false, st));
+  else if (kernel == 6)
+    CK(x, launch_tile_chain(x->D, x->B, *tile_maps(x), x->layers[layer],
+                            layer + 1 < x->cfg.n_layers ? &x->layers[layer + 1] : nullptr, layer,
+                            sel, M, st));
   else
     CK(x, launch_layer_part(x->D, x->B, x->cfg.dtype, x->layers[layer], tile_maps(x), layer,
                             kernel, sel, M, st));

@@ -783,6 +783,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_stream(const StreamArgs a, cons
 // ------------------------------------------------------------- launchers
 
 bool g_pdl_enabled = true;
+bool g_chain_enabled = true;
 thread_local bool g_pdl_ok = true;
 
 static Geom make_geom(const Dims& D, int N, int K, int elt, int map) {

@@ -35,6 +35,11 @@ cudaError_t prepare_tile_kernels();
 size_t tile_part_floats(int num_sms);
 cudaError_t launch_tile_part(const Dims& D, const Bufs& B, const TileMaps& tm, const LayerW& w,
                              int layer, int part, RowSel sel, int mrows, cudaStream_t st);
+// One launch of a layer's O projection, gate/up and down (and, with next, the
+// next layer's QKV) as the phases of one persistent kernel.
+cudaError_t launch_tile_chain(const Dims& D, const Bufs& B, const TileMaps& tm, const LayerW& w,
+                              const LayerW* next, int layer, RowSel sel, int mrows,
+                              cudaStream_t st);
 cudaError_t launch_tile_head(const Dims& D, const Bufs& B, const TileMaps& tm,
                              const CUtensorMap& lm, const void* final_norm, int topk,
                              bool write_logits, RowSel sel, int mrows, cudaStream_t st);

@@ -95,6 +95,9 @@ __device__ __forceinline__ void named_sync(int id, int threads) {
 // kernel after a conditional node or at the start of a body keeps a full
 // dependency, and set again after every launch.
 extern bool g_pdl_enabled;
+// bf16 layer passes run O, gate/up, down and the next QKV as one persistent
+// launch (env SSD_NO_CHAIN=1: one launch per matrix, same results bit for bit)
+extern bool g_chain_enabled;
 extern thread_local bool g_pdl_ok;
 
 template <typename Kern, typename... Args>

@@ -33,6 +33,7 @@
 #include <cudaTypedefs.h>
 
 #include <mutex>
+#include <type_traits>
 
 #include "headpart.cuh"
 #include "kernels.h"
@@ -238,12 +239,12 @@ __device__ __forceinline__ void t_pair(const TArgs& a, int tile, int s, int t, i
     const int r0 = trow(a.g, tile, s), r1 = trow(a.g, tile, s + 128);
     float* hm = a.B.h + (size_t)t * D.d;
     if (r0 >= 0) {
-      const float h = hm[r0] + v0;
+      const float h = __ldcg(hm + r0) + v0;  // L2: rows a previous phase wrote
       hm[r0] = h;
       ss = fmaf(h, h, ss);
     }
     if (r1 >= 0) {
-      const float h = hm[r1] + v1;
+      const float h = __ldcg(hm + r1) + v1;
       hm[r1] = h;
       ss = fmaf(h, h, ss);
     }
@@ -274,309 +275,286 @@ __device__ __forceinline__ void t_head_token(const TArgs& a, int tile, int s, in
 
 }  // namespace
 
-// ------------------------------------------------------------ the kernel
+// ------------------------------------------------------------ the kernels
 
+// Shared-memory views of one block (layout TL<TP, HEAD>).
+template <int TP, bool HEAD>
+struct Blk {
+  using S = TL<TP, HEAD>;
+  unsigned char* smem;
+  uint64_t *full, *xfull, *empty, *bfull, *accfull, *accempty, *drain;
+  uint32_t* tslot;
+  int* sflag;
+  float *srs, *red;
+  HeadPart *run, *spl, *comb;
+
+  __device__ explicit Blk(unsigned char* raw) {
+    smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(raw) + 1023) &
+                                            ~static_cast<uintptr_t>(1023));
+    full = reinterpret_cast<uint64_t*>(smem + S::bars);  // weights landed
+    xfull = full + S::NS;                                // input slice landed
+    empty = xfull + S::NS;                               // slot released by the MMAs
+    bfull = empty + S::NS;                               // operand tile written
+    accfull = bfull + S::NS;
+    accempty = accfull + 2;
+    drain = accempty + 2;
+    tslot = reinterpret_cast<uint32_t*>(smem + S::tslot);
+    sflag = reinterpret_cast<int*>(smem + S::flag);
+    srs = reinterpret_cast<float*>(smem + S::rs);
+    red = reinterpret_cast<float*>(smem + S::red);
+    run = reinterpret_cast<HeadPart*>(smem + S::run);
+    spl = reinterpret_cast<HeadPart*>(smem + S::spl);
+    comb = reinterpret_cast<HeadPart*>(smem + S::comb);
+  }
+
+  // barriers (thread 0), TMEM allocation (the MMA warp); every thread waits
+  __device__ uint32_t setup(int warp, int mma_warp) {
+    if (threadIdx.x == 0) {
+      for (int i = 0; i < S::NS; ++i) {
+        mbar_init(&full[i], 1);
+        mbar_init(&xfull[i], 1);
+        mbar_init(&empty[i], 1);         // MMA commit
+        mbar_init(&bfull[i], kWorkers);  // operand tile written
+      }
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(&accfull[i], 1);
+        mbar_init(&accempty[i], kWorkers);
+      }
+      mbar_init(drain, 1);
+      mbar_init_fence();
+    }
+    if (warp == mma_warp) tc_alloc(tslot, S::kCols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    return *tslot;
+  }
+
+  // workers: zeroed operand tiles (rows past M stay zero), empty statistics
+  __device__ void clear_operands(int tid) {
+    uint4* z = reinterpret_cast<uint4*>(smem + S::bt);
+    for (int i = tid; i < S::NS * S::BB / 16; i += kWThreads) z[i] = make_uint4(0, 0, 0, 0);
+    if constexpr (HEAD)
+      for (int i = tid; i < kWorkers * kLT; i += kWThreads) part_empty(run[i]);
+    fence_proxy_async_smem();
+    named_sync(1, kWThreads);
+  }
+};
+
+// MMA issue (one thread) for the block's units [u_begin, u_begin + n) of one
+// matrix: per unit both 128-row halves times four K-steps of 16, high and low
+// parts as one N = 2 TP operand.  gi0 is the block's count of units before
+// this matrix (ring slot and phase parity continue across the matrices of a
+// chain), tc the running tile count (double-buffered TMEM accumulator).
+template <int TP, bool HEAD>
+__device__ bool mma_units(const Blk<TP, HEAD>& k, const TGeom& g, int u_begin, int n, int gi0,
+                          int& tc, uint32_t tmem) {
+  using S = TL<TP, HEAD>;
+  constexpr int NS = S::NS, N = S::N;
+  constexpr uint32_t idesc = idesc_bf16_f32(128, N);
+  for (int i = 0; i < n; ++i) {
+    const int gi = gi0 + i;
+    const int u = u_begin + i;
+    const int slot = gi % NS;
+    const uint32_t ph = (uint32_t)(gi / NS) & 1u;
+    const bool first = (i == 0) || (u % g.nks == 0);
+    const bool last = (i == n - 1) || ((u + 1) % g.nks == 0);
+    if (first) {
+      ++tc;
+      if (!mbar_wait(&k.accempty[tc & 1], ((uint32_t)(tc >> 1) & 1u) ^ 1u)) return false;
+    }
+    if (!mbar_wait(&k.full[slot], ph) || !mbar_wait(&k.bfull[slot], ph)) return false;
+    tc_fence_after();
+    const uint32_t abase = smem_u32(k.smem + S::ring + (size_t)slot * kWBytes);
+    const uint32_t bbase = smem_u32(k.smem + S::bt + (size_t)slot * S::BB);
+    const uint32_t dbase = tmem + (uint32_t)((tc & 1) * 2 * N);
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+      for (int kk = 0; kk < kKC / 16; ++kk)
+        tc_mma_bf16(dbase + h * N, sdesc_k128(abase + h * (kWBytes / 2) + kk * 32),
+                    sdesc_k128(bbase + kk * 32), idesc, !first || kk > 0);
+    tc_commit(&k.empty[slot]);
+    if (last) tc_commit(&k.accfull[tc & 1]);
+  }
+  return true;
+}
+
+// Workers (eight warps) for the block's units of one matrix: operand tiles
+// from the input slices, then the fused epilogue of every tile.  The RMSNorm
+// scale of the input rows is read first (from the sum-of-squares parts).
 template <int TP, int KIND, bool NORM>
-__global__ void __launch_bounds__(kTThreads, 1)
-    k_tile(const __grid_constant__ CUtensorMap wmap, const __grid_constant__ CUtensorMap xmap,
-           const TArgs a) {
+__device__ void worker_units(const TArgs& a, const Blk<TP, KIND == kKHead>& k, uint32_t tmem,
+                             int u_begin, int n, int gi0, int& tc, bool& ok, int pos0, int M) {
   using S = TL<TP, KIND == kKHead>;
   constexpr int NS = S::NS, N = S::N;
   constexpr int LTN = TP / 2;                 // tokens per parity group read back
   constexpr int LTR = LTN < kLT ? LTN : kLT;  // ... of which can be rows (t < kMaxM)
-  extern __shared__ unsigned char smem_raw[];
-  unsigned char* smem = reinterpret_cast<unsigned char*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::bars);  // weights landed
-  uint64_t* xfull = full + NS;                                   // input slice landed
-  uint64_t* empty = xfull + NS;
-  uint64_t* bfull = empty + NS;
-  uint64_t* accfull = bfull + NS;
-  uint64_t* accempty = accfull + 2;
-  uint64_t* drain = accempty + 2;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + S::tslot);
-  int* sflag = reinterpret_cast<int*>(smem + S::flag);
-  float* srs = reinterpret_cast<float*>(smem + S::rs);
-  float* red = reinterpret_cast<float*>(smem + S::red);
-  HeadPart* run = reinterpret_cast<HeadPart*>(smem + S::run);
-  HeadPart* spl = reinterpret_cast<HeadPart*>(smem + S::spl);
-  HeadPart* comb = reinterpret_cast<HeadPart*>(smem + S::comb);
-
   const TGeom& g = a.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
-  const int u_begin = t_start(g, blockIdx.x), u_end = t_start(g, blockIdx.x + 1);
-  const int n = (int)(u_end - u_begin);
-
-  if (tid == 0) {
-    for (int i = 0; i < NS; ++i) {
-      mbar_init(&full[i], 1);
-      mbar_init(&xfull[i], 1);
-      mbar_init(&empty[i], 1);         // MMA commit
-      mbar_init(&bfull[i], kWorkers);  // operand tile written
-    }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&accfull[i], 1);
-      mbar_init(&accempty[i], kWorkers);
-    }
-    mbar_init(drain, 1);
-    mbar_init_fence();
-  }
-  if (warp == kMmaWarp) tc_alloc(tslot, S::kCols);
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tslot;
-  pdl_launch_dependents();
-
-  if (warp == kTmaWarp) {
-    // ---------------- TMA: weights need nothing from earlier kernels, the
-    // input slices wait for them
-    if (lane == 0 && n > 0) {
-      const uint64_t pol = evict_first_policy();
-      tma_prefetch_desc(&wmap);
-      tma_prefetch_desc(&xmap);
-      auto issue_w = [&](int i) -> bool {
-        const int slot = i % NS;
-        if (!mbar_wait(&empty[slot], ((uint32_t)(i / NS) & 1u) ^ 1u)) return false;
-        const int u = u_begin + i;
-        const int tile = u / g.nks, kc = u - tile * g.nks;
-        mbar_arrive_expect_tx(&full[slot], (uint32_t)kWBytes);
-        unsigned char* dst = smem + S::ring + (size_t)slot * kWBytes;
-#pragma unroll
-        for (int b = 0; b < 4; ++b)
-          tma_load_2d(dst + b * kBoxBytes, &wmap, kc * kKC, box_row(g, tile, b), &full[slot], pol);
-        return true;
-      };
-      const int npre = n < NS ? n : NS;
-      bool ok = true;
-      for (int i = 0; i < npre && ok; ++i) ok = issue_w(i);
-      pdl_wait();
-      const int K = g.K;
-      for (int i = 0; i < n && ok; ++i) {
-        if (i >= npre) ok = issue_w(i);
-        if (!ok) break;
-        const int slot = i % NS;
-        const int kc = (int)((u_begin + i) % g.nks);
-        unsigned char* xdst = smem + S::xs + (size_t)slot * S::XS;
-        const int cols = min(kKC, K - kc * kKC);
-        const uint32_t gbytes = NORM ? (uint32_t)cols * 2u : 0u;
-        mbar_arrive_expect_tx(&xfull[slot], (uint32_t)S::XB + gbytes);
-        tma_load_2d(xdst, &xmap, kc * kKC, 0, &xfull[slot], pol);
-        if (NORM) bulk_g2s(xdst + S::XB, a.gnorm + (size_t)kc * kKC, gbytes, &xfull[slot], pol);
-      }
-      if (!ok) flag_timeout(a.B);
-      // every copy has landed before the block exits
-      for (int k = n > NS ? n - NS : 0; k < n; ++k) {
-        mbar_wait(&full[k % NS], (uint32_t)(k / NS) & 1u);
-        mbar_wait(&xfull[k % NS], (uint32_t)(k / NS) & 1u);
-      }
-    }
-  } else if (warp == kMmaWarp) {
-    // ---------------- MMA issue (one thread): per unit, both 128-row halves
-    // times four K-steps of 16, high and low parts as one N = 2 TP operand
-    if (lane == 0 && n > 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(128, N);
-      bool ok = true;
-      int tc = -1;
-      for (int i = 0; i < n && ok; ++i) {
-        const int u = u_begin + i;
-        const int slot = i % NS;
-        const uint32_t ph = (uint32_t)(i / NS) & 1u;
-        const bool first = (i == 0) || (u % g.nks == 0);
-        const bool last = (i == n - 1) || ((u + 1) % g.nks == 0);
-        if (first) {
-          ++tc;
-          ok = mbar_wait(&accempty[tc & 1], ((uint32_t)(tc >> 1) & 1u) ^ 1u);
-        }
-        ok = ok && mbar_wait(&full[slot], ph) && mbar_wait(&bfull[slot], ph);
-        if (!ok) break;
-        tc_fence_after();
-        const uint32_t abase = smem_u32(smem + S::ring + (size_t)slot * kWBytes);
-        const uint32_t bbase = smem_u32(smem + S::bt + (size_t)slot * S::BB);
-        const uint32_t dbase = tmem + (uint32_t)((tc & 1) * 2 * N);
-#pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-          for (int kk = 0; kk < kKC / 16; ++kk)
-            tc_mma_bf16(dbase + h * N, sdesc_k128(abase + h * (kWBytes / 2) + kk * 32),
-                        sdesc_k128(bbase + kk * 32), idesc, !first || kk > 0);
-        tc_commit(&empty[slot]);
-        if (last) tc_commit(&accfull[tc & 1]);
-      }
-      if (!ok) flag_timeout(a.B);
-      // every MMA has completed before TMEM is released
-      tc_commit(drain);
-      if (!mbar_wait(drain, 0)) flag_timeout(a.B);
-    }
-  } else {
-    // ---------------- workers: operand tiles and epilogues
-    pdl_wait();
-    int pos0, M;
-    resolve_rows(a.B.ctl, a.sel, pos0, M);
-    if (M > TP) M = TP;  // the launcher picks TP >= M
-    if (tid < 32) {
-      // RMSNorm scale of row tid: the input's sum of squares is kept as parts
-      // of 256 elements, added here in part order
-      float r = 1.f;
-      if (a.ss_in >= 0 && tid < M) {
-        const float* sp = a.B.ss_part + (size_t)a.ss_in * a.D.ss_nt * kMaxM + tid;
-        float sum = 0.f;
+  float* srs = k.srs;
+  float* red = k.red;
+  int* sflag = k.sflag;
+  HeadPart* run = k.run;
+  HeadPart* spl = k.spl;
+  if (tid < 32) {
+    // RMSNorm scale of row tid: the input's sum of squares is kept as parts
+    // of 256 elements, added here in part order
+    float r = 1.f;
+    if (a.ss_in >= 0 && tid < M) {
+      const float* sp = a.B.ss_part + (size_t)a.ss_in * a.D.ss_nt * kMaxM + tid;
+      float sum = 0.f;
 #pragma unroll 8
-        for (int c = 0; c < a.D.ss_nt; ++c) sum += __ldcg(&sp[(size_t)c * kMaxM]);
-        r = 1.0f / sqrtf(sum / (float)g.K + a.D.eps);
-      }
-      srs[tid] = r;
+      for (int c = 0; c < a.D.ss_nt; ++c) sum += __ldcg(&sp[(size_t)c * kMaxM]);
+      r = 1.0f / sqrtf(sum / (float)g.K + a.D.eps);
     }
-    {
-      uint4* z = reinterpret_cast<uint4*>(smem + S::bt);
-      for (int i = tid; i < NS * S::BB / 16; i += kWThreads) z[i] = make_uint4(0, 0, 0, 0);
-      if constexpr (KIND == kKHead)
-        for (int i = tid; i < kWorkers * kLT; i += kWThreads) part_empty(run[i]);
+    srs[tid] = r;
+  }
+  named_sync(1, kWThreads);
+  const int q = warp & 3, grp = warp >> 2;
+  const int srow = 32 * q + lane;  // stage row of half 0 (half 1: + 128)
+  float rs_t[LTN];
+#pragma unroll
+  for (int lt = 0; lt < LTN; ++lt) rs_t[lt] = srs[2 * lt + grp];
+  const int u_end = u_begin + n;
+  const int first_tile = u_begin / g.nks;
+
+  // Residual kernels: sum of squares of the tile's 256 updated rows per
+  // token (fixed order: lanes, then the four row quarters), one part of the
+  // next RMSNorm's input
+  auto tile_ss = [&](const float (&ssv)[LTN], int tile) {
+#pragma unroll
+    for (int lt = 0; lt < LTR; ++lt) {
+      const float sw = warp_sum(ssv[lt]);
+      if (lane == 0) red[warp * kLT + lt] = sw;
     }
-    fence_proxy_async_smem();
     named_sync(1, kWThreads);
-    const int q = warp & 3, grp = warp >> 2;
-    const int srow = 32 * q + lane;  // stage row of half 0 (half 1: + 128)
-    float rs_t[LTN];
-#pragma unroll
-    for (int lt = 0; lt < LTN; ++lt) rs_t[lt] = srs[2 * lt + grp];
-    bool ok = true;
-    const int first_tile = (int)(u_begin / g.nks);
+    if (tid < M) {
+      float sum = 0.f;
+      for (int qq = 0; qq < 4; ++qq) sum += red[((tid & 1) * 4 + qq) * kLT + (tid >> 1)];
+      a.B.ss_part[((size_t)a.which * a.D.ss_nt + tile) * kMaxM + tid] = sum;
+    }
+    named_sync(1, kWThreads);
+  };
 
-    // Residual kernels: sum of squares of the tile's 256 updated rows per
-    // token (fixed order: lanes, then the four row quarters), one part of the
-    // next RMSNorm's input
-    auto tile_ss = [&](const float (&ssv)[LTN], int tile) {
+  // per-tile epilogue: TMEM -> registers (high + low parts) -> fused epilogue
+  auto epilogue = [&](int tile, int tcv) {
+    const int buf = tcv & 1;
+    if (ok) {
+      const bool w = __all_sync(0xffffffffu, mbar_wait(&k.accfull[buf], (uint32_t)(tcv >> 1) & 1u));
+      if (!w) {
+        if (lane == 0) flag_timeout(a.B);
+        ok = false;
+      }
+    }
+    tc_fence_after();
+    float v[2][TP];
 #pragma unroll
-      for (int lt = 0; lt < LTR; ++lt) {
-        const float sw = warp_sum(ssv[lt]);
-        if (lane == 0) red[warp * kLT + lt] = sw;
-      }
-      named_sync(1, kWThreads);
-      if (tid < M) {
-        float sum = 0.f;
-        for (int qq = 0; qq < 4; ++qq) sum += red[((tid & 1) * 4 + qq) * kLT + (tid >> 1)];
-        a.B.ss_part[((size_t)a.which * a.D.ss_nt + tile) * kMaxM + tid] = sum;
-      }
-      named_sync(1, kWThreads);
-    };
-
-    // per-tile epilogue: TMEM -> registers (high + low parts) -> fused epilogue
-    auto epilogue = [&](int tile, int tc) {
-      const int buf = tc & 1;
-      if (ok) {
-        const bool w = __all_sync(0xffffffffu, mbar_wait(&accfull[buf], (uint32_t)(tc >> 1) & 1u));
-        if (!w) {
-          if (lane == 0) flag_timeout(a.B);
-          ok = false;
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+      for (int c = 0; c < TP / 8; ++c) {
+        float hi8[8], lo8[8];
+        if (ok) {
+          const uint32_t col =
+              tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * 2 * N + h * N + c * 8);
+          tc_ld8(col, hi8);
+          tc_ld8(col + TP, lo8);
+        } else {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) hi8[e] = lo8[e] = 0.f;
         }
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[h][c * 8 + e] = hi8[e] + lo8[e];
       }
-      tc_fence_after();
-      float v[2][TP];
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&k.accempty[buf]);
+    const int t0 = tile * g.nks, t1 = t0 + g.nks;
+    if (t0 >= u_begin && t1 <= u_end) {
+      float ssv[LTN];
 #pragma unroll
-      for (int h = 0; h < 2; ++h)
-#pragma unroll
-        for (int c = 0; c < TP / 8; ++c) {
-          float hi8[8], lo8[8];
-          if (ok) {
-            const uint32_t col = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * 2 * N + h * N + c * 8);
-            tc_ld8(col, hi8);
-            tc_ld8(col + TP, lo8);
-          } else {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) hi8[e] = lo8[e] = 0.f;
-          }
-#pragma unroll
-          for (int e = 0; e < 8; ++e) v[h][c * 8 + e] = hi8[e] + lo8[e];
-        }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&accempty[buf]);
-      const int t0 = tile * g.nks, t1 = t0 + g.nks;
-      if (t0 >= u_begin && t1 <= u_end) {
-        float ssv[LTN];
-#pragma unroll
-        for (int lt = 0; lt < LTN; ++lt) ssv[lt] = 0.f;
-#pragma unroll
-        for (int lt = 0; lt < LTN; ++lt) {
-          const int t = 2 * lt + grp;
-          if (t >= M) break;
-          const float v0 = grp ? v[0][2 * lt + 1] : v[0][2 * lt];
-          const float v1 = grp ? v[1][2 * lt + 1] : v[1][2 * lt];
-          if constexpr (KIND == kKHead)
-            t_head_token(a, tile, srow, t, rs_t[lt], v0, v1, &run[warp * kLT + lt], lane);
-          else
-            t_pair<KIND>(a, tile, srow, t, pos0, rs_t[lt], v0, v1, ssv[lt]);
-        }
-        if constexpr (KIND == kKResid) tile_ss(ssv, tile);
-        return;
-      }
-      // shared with neighbouring blocks: publish this block's partial sums
-      const int slot2 = tile == first_tile ? 0 : 1;
-      float* mine = a.B.gpart + ((size_t)blockIdx.x * 2 + slot2) * 2 * kMaxM * 128;
+      for (int lt = 0; lt < LTN; ++lt) ssv[lt] = 0.f;
 #pragma unroll
       for (int lt = 0; lt < LTN; ++lt) {
         const int t = 2 * lt + grp;
         if (t >= M) break;
-        mine[(size_t)t * 128 + srow] = grp ? v[0][2 * lt + 1] : v[0][2 * lt];
-        mine[(size_t)(kMaxM + t) * 128 + srow] = grp ? v[1][2 * lt + 1] : v[1][2 * lt];
+        const float v0 = grp ? v[0][2 * lt + 1] : v[0][2 * lt];
+        const float v1 = grp ? v[1][2 * lt + 1] : v[1][2 * lt];
+        if constexpr (KIND == kKHead)
+          t_head_token(a, tile, srow, t, rs_t[lt], v0, v1, &run[warp * kLT + lt], lane);
+        else
+          t_pair<KIND>(a, tile, srow, t, pos0, rs_t[lt], v0, v1, ssv[lt]);
       }
-      __threadfence();
-      named_sync(1, kWThreads);
-      const int b0 = t_block_of(g, t0), b1 = t_block_of(g, t1 - 1);
-      if (tid == 0) {
-        int contrib = 0;
-        for (int b = b0; b <= b1; ++b) contrib += t_start(g, b) < t_start(g, b + 1);
-        *sflag = atomicAdd(&a.B.tile_counter[tile], 1u) == (unsigned)(contrib - 1);
-      }
-      named_sync(1, kWThreads);
-      if (!*sflag) return;
-      __threadfence();
-      if (tid == 0) a.B.tile_counter[tile] = 0u;
-      float ss_sp[LTN];
+      if constexpr (KIND == kKResid) tile_ss(ssv, tile);
+      return;
+    }
+    // shared with neighbouring blocks: publish this block's partial sums
+    const int slot2 = tile == first_tile ? 0 : 1;
+    float* mine = a.B.gpart + ((size_t)blockIdx.x * 2 + slot2) * 2 * kMaxM * 128;
 #pragma unroll
-      for (int lt = 0; lt < LTN; ++lt) ss_sp[lt] = 0.f;
-      if constexpr (KIND == kKHead) {
-        if (lane == 0)
-          for (int lt = 0; lt < kLT; ++lt) part_empty(spl[warp * kLT + lt]);
-        __syncwarp();
-      }
-      // Partial sums of the contributors, added in block order (independent of
-      // who finishes last).  The loads of several contributors (and all
-      // tokens) are issued before any is used, so the fix-up costs a few L2
-      // round trips rather than one per contributor and token.  Unused slots
-      // read block 0's partials (valid memory) and add zero.
-      constexpr int GB = LTN <= 4 ? 4 : (LTN <= 8 ? 2 : 1);
-      float u0[LTN], u1[LTN];
+    for (int lt = 0; lt < LTN; ++lt) {
+      const int t = 2 * lt + grp;
+      if (t >= M) break;
+      mine[(size_t)t * 128 + srow] = grp ? v[0][2 * lt + 1] : v[0][2 * lt];
+      mine[(size_t)(kMaxM + t) * 128 + srow] = grp ? v[1][2 * lt + 1] : v[1][2 * lt];
+    }
+    __threadfence();
+    named_sync(1, kWThreads);
+    const int b0 = t_block_of(g, t0), b1 = t_block_of(g, t1 - 1);
+    if (tid == 0) {
+      int contrib = 0;
+      for (int b = b0; b <= b1; ++b) contrib += t_start(g, b) < t_start(g, b + 1);
+      *sflag = atomicAdd(&a.B.tile_counter[tile], 1u) == (unsigned)(contrib - 1);
+    }
+    named_sync(1, kWThreads);
+    if (!*sflag) return;
+    __threadfence();
+    if (tid == 0) a.B.tile_counter[tile] = 0u;
+    float ss_sp[LTN];
 #pragma unroll
-      for (int lt = 0; lt < LTN; ++lt) u0[lt] = u1[lt] = 0.f;
-      if (M == 1) {
-        // one token (drafting, autoregressive steps): sixteen contributors per round
-        for (int b = grp == 0 ? b0 : b1 + 1; b <= b1; b += 16) {
-          float c0[16], c1[16];
+    for (int lt = 0; lt < LTN; ++lt) ss_sp[lt] = 0.f;
+    if constexpr (KIND == kKHead) {
+      if (lane == 0)
+        for (int lt = 0; lt < kLT; ++lt) part_empty(spl[warp * kLT + lt]);
+      __syncwarp();
+    }
+    // Partial sums of the contributors, added in block order (independent of
+    // who finishes last).  The loads of several contributors (and all
+    // tokens) are issued before any is used, so the fix-up costs a few L2
+    // round trips rather than one per contributor and token.  Unused slots
+    // read block 0's partials (valid memory) and add zero.
+    constexpr int GB = LTN <= 4 ? 4 : (LTN <= 8 ? 2 : 1);
+    float u0[LTN], u1[LTN];
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const int bb = b + j;
-            bool use = false;
-            int sl = 0;
-            if (bb <= b1) {
-              const int sb = t_start(g, bb);
-              use = sb != t_start(g, bb + 1);
-              sl = tile == (int)(sb / g.nks) ? 0 : 1;
-            }
-            const float* p = a.B.gpart + ((size_t)(use ? bb : 0) * 2 + sl) * 2 * kMaxM * 128;
-            const float x0 = __ldcg(&p[srow]);
-            const float x1 = __ldcg(&p[(size_t)kMaxM * 128 + srow]);
-            c0[j] = use ? x0 : 0.f;
-            c1[j] = use ? x1 : 0.f;
+    for (int lt = 0; lt < LTN; ++lt) u0[lt] = u1[lt] = 0.f;
+    if (M == 1) {
+      // one token (drafting, autoregressive steps): sixteen contributors per round
+      for (int b = grp == 0 ? b0 : b1 + 1; b <= b1; b += 16) {
+        float c0[16], c1[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const int bb = b + j;
+          bool use = false;
+          int sl = 0;
+          if (bb <= b1) {
+            const int sb = t_start(g, bb);
+            use = sb != t_start(g, bb + 1);
+            sl = tile == (int)(sb / g.nks) ? 0 : 1;
           }
-#pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            u0[0] += c0[j];
-            u1[0] += c1[j];
-          }
+          const float* p = a.B.gpart + ((size_t)(use ? bb : 0) * 2 + sl) * 2 * kMaxM * 128;
+          const float x0 = __ldcg(&p[srow]);
+          const float x1 = __ldcg(&p[(size_t)kMaxM * 128 + srow]);
+          c0[j] = use ? x0 : 0.f;
+          c1[j] = use ? x1 : 0.f;
         }
-      } else for (int b = b0; b <= b1; b += GB) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          u0[0] += c0[j];
+          u1[0] += c1[j];
+        }
+      }
+    } else
+      for (int b = b0; b <= b1; b += GB) {
         float c0[GB][LTN], c1[GB][LTN];
 #pragma unroll
         for (int j = 0; j < GB; ++j) {
@@ -608,90 +586,173 @@ __global__ void __launch_bounds__(kTThreads, 1)
           }
       }
 #pragma unroll
-      for (int lt = 0; lt < LTN; ++lt) {
-        const int t = 2 * lt + grp;
-        if (t >= M) break;
-        if constexpr (KIND == kKHead)
-          t_head_token(a, tile, srow, t, rs_t[lt], u0[lt], u1[lt], &spl[warp * kLT + lt], lane);
-        else
-          t_pair<KIND>(a, tile, srow, t, pos0, rs_t[lt], u0[lt], u1[lt], ss_sp[lt]);
-      }
-      // the split tile's statistics: residual sums of squares as the tile's
-      // part; exit-head statistics to the split slot of its first block
-      if constexpr (KIND == kKResid) {
-        tile_ss(ss_sp, tile);
-      } else if constexpr (KIND == kKHead) {
-        named_sync(1, kWThreads);
-        if (tid < M) {
-          HeadPart p;
-          part_empty(p);
-          for (int qq = 0; qq < 4; ++qq) part_merge(p, spl[((tid & 1) * 4 + qq) * kLT + (tid >> 1)]);
-          static_cast<HeadPart*>(a.B.head_part)[((size_t)kMaxBlocksDev + b0) * kMaxM + tid] = p;
-        }
-        named_sync(1, kWThreads);
-      }
-    };
-
-    int tc = -1;
-    int prev_tile = -1;
-    for (int i = 0; i < n; ++i) {
-      const int u = u_begin + i;
-      const int slot = i % NS;
-      const int tile = u / g.nks, kc = u - tile * g.nks;
-      if (i == 0 || kc == 0) ++tc;
-      // operand tile of unit i, built while its weights are still in flight:
-      // the slot's previous use was released before its copies were issued,
-      // so only the input slice's arrival is waited for
-      if (ok) {
-        const bool w = __all_sync(0xffffffffu, mbar_wait(&xfull[slot], (uint32_t)(i / NS) & 1u));
-        if (!w) {
-          if (lane == 0) flag_timeout(a.B);
-          ok = false;
-        }
-      }
-      if (ok) {
-        const unsigned char* xs = smem + S::xs + (size_t)slot * S::XS;
-        unsigned char* bt = smem + S::bt + (size_t)slot * S::BB;
-        const int kvalid = g.K - kc * kKC;
-        for (int task = tid; task < M * 8; task += kWThreads) {
-          const int m = task >> 3, j = task & 7;
-          const float4 x0 = *reinterpret_cast<const float4*>(xs + m * (kKC * 4) + j * 32);
-          const float4 x1 = *reinterpret_cast<const float4*>(xs + m * (kKC * 4) + j * 32 + 16);
-          float xv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-          if (NORM) {
-            const uint4 gq = *reinterpret_cast<const uint4*>(xs + S::XB + j * 16);
-            float gv[8];
-            Elem<__nv_bfloat16>::unpack(gq, gv);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) xv[e] *= gv[e];
-          }
-#pragma unroll
-          for (int e = 0; e < 8; ++e)
-            if (j * 8 + e >= kvalid) xv[e] = 0.f;
-          uint32_t hi[4], lo[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const __nv_bfloat16 h0 = __float2bfloat16_rn(xv[2 * e]);
-            const __nv_bfloat16 h1 = __float2bfloat16_rn(xv[2 * e + 1]);
-            hi[e] = pack_bf16(h0, h1);
-            lo[e] = pack_bf16(__float2bfloat16_rn(xv[2 * e] - __bfloat162float(h0)),
-                              __float2bfloat16_rn(xv[2 * e + 1] - __bfloat162float(h1)));
-          }
-          *reinterpret_cast<uint4*>(bt + swz(m, j)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-          *reinterpret_cast<uint4*>(bt + swz(TP + m, j)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
-        }
-        fence_proxy_async_smem();
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bfull[slot]);
-      // epilogue of the tile the previous unit completed
-      if (i > 0 && kc == 0) epilogue(prev_tile, tc - 1);
-      prev_tile = tile;
+    for (int lt = 0; lt < LTN; ++lt) {
+      const int t = 2 * lt + grp;
+      if (t >= M) break;
+      if constexpr (KIND == kKHead)
+        t_head_token(a, tile, srow, t, rs_t[lt], u0[lt], u1[lt], &spl[warp * kLT + lt], lane);
+      else
+        t_pair<KIND>(a, tile, srow, t, pos0, rs_t[lt], u0[lt], u1[lt], ss_sp[lt]);
     }
-    if (n > 0) epilogue(prev_tile, tc);
+    // the split tile's statistics: residual sums of squares as the tile's
+    // part; exit-head statistics to the split slot of its first block
+    if constexpr (KIND == kKResid) {
+      tile_ss(ss_sp, tile);
+    } else if constexpr (KIND == kKHead) {
+      named_sync(1, kWThreads);
+      if (tid < M) {
+        HeadPart p;
+        part_empty(p);
+        for (int qq = 0; qq < 4; ++qq) part_merge(p, spl[((tid & 1) * 4 + qq) * kLT + (tid >> 1)]);
+        static_cast<HeadPart*>(a.B.head_part)[((size_t)kMaxBlocksDev + b0) * kMaxM + tid] = p;
+      }
+      named_sync(1, kWThreads);
+    }
+  };
+
+  int prev_tile = -1;
+  for (int i = 0; i < n; ++i) {
+    const int gi = gi0 + i;
+    const int u = u_begin + i;
+    const int slot = gi % NS;
+    const int tile = u / g.nks, kc = u - tile * g.nks;
+    if (i == 0 || kc == 0) ++tc;
+    // operand tile of unit i, built while its weights are still in flight:
+    // the slot's previous use was released before its copies were issued,
+    // so only the input slice's arrival is waited for
+    if (ok) {
+      const bool w = __all_sync(0xffffffffu, mbar_wait(&k.xfull[slot], (uint32_t)(gi / NS) & 1u));
+      if (!w) {
+        if (lane == 0) flag_timeout(a.B);
+        ok = false;
+      }
+    }
+    if (ok) {
+      const unsigned char* xs = k.smem + S::xs + (size_t)slot * S::XS;
+      unsigned char* bt = k.smem + S::bt + (size_t)slot * S::BB;
+      const int kvalid = g.K - kc * kKC;
+      for (int task = tid; task < M * 8; task += kWThreads) {
+        const int m = task >> 3, j = task & 7;
+        const float4 x0 = *reinterpret_cast<const float4*>(xs + m * (kKC * 4) + j * 32);
+        const float4 x1 = *reinterpret_cast<const float4*>(xs + m * (kKC * 4) + j * 32 + 16);
+        float xv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+        if (NORM) {
+          const uint4 gq = *reinterpret_cast<const uint4*>(xs + S::XB + j * 16);
+          float gv[8];
+          Elem<__nv_bfloat16>::unpack(gq, gv);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) xv[e] *= gv[e];
+        }
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+          if (j * 8 + e >= kvalid) xv[e] = 0.f;
+        uint32_t hi[4], lo[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const __nv_bfloat16 h0 = __float2bfloat16_rn(xv[2 * e]);
+          const __nv_bfloat16 h1 = __float2bfloat16_rn(xv[2 * e + 1]);
+          hi[e] = pack_bf16(h0, h1);
+          lo[e] = pack_bf16(__float2bfloat16_rn(xv[2 * e] - __bfloat162float(h0)),
+                            __float2bfloat16_rn(xv[2 * e + 1] - __bfloat162float(h1)));
+        }
+        *reinterpret_cast<uint4*>(bt + swz(m, j)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+        *reinterpret_cast<uint4*>(bt + swz(TP + m, j)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+      }
+      fence_proxy_async_smem();
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&k.bfull[slot]);
+    // epilogue of the tile the previous unit completed
+    if (i > 0 && kc == 0) epilogue(prev_tile, tc - 1);
+    prev_tile = tile;
+  }
+  if (n > 0) epilogue(prev_tile, tc);
+}
+
+template <int TP, int KIND, bool NORM>
+__global__ void __launch_bounds__(kTThreads, 1)
+    k_tile(const __grid_constant__ CUtensorMap wmap, const __grid_constant__ CUtensorMap xmap,
+           const TArgs a) {
+  using S = TL<TP, KIND == kKHead>;
+  constexpr int NS = S::NS;
+  extern __shared__ unsigned char smem_raw[];
+  Blk<TP, KIND == kKHead> k(smem_raw);
+  unsigned char* smem = k.smem;
+  const TGeom& g = a.g;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
+  const int u_begin = t_start(g, blockIdx.x), u_end = t_start(g, blockIdx.x + 1);
+  const int n = u_end - u_begin;
+  const uint32_t tmem = k.setup(warp, kMmaWarp);
+  pdl_launch_dependents();
+
+  if (warp == kTmaWarp) {
+    // ---------------- TMA: weights need nothing from earlier kernels, the
+    // input slices wait for them
+    if (lane == 0 && n > 0) {
+      const uint64_t pol = evict_first_policy();
+      tma_prefetch_desc(&wmap);
+      tma_prefetch_desc(&xmap);
+      auto issue_w = [&](int i) -> bool {
+        const int slot = i % NS;
+        if (!mbar_wait(&k.empty[slot], ((uint32_t)(i / NS) & 1u) ^ 1u)) return false;
+        const int u = u_begin + i;
+        const int tile = u / g.nks, kc = u - tile * g.nks;
+        mbar_arrive_expect_tx(&k.full[slot], (uint32_t)kWBytes);
+        unsigned char* dst = smem + S::ring + (size_t)slot * kWBytes;
+#pragma unroll
+        for (int b = 0; b < 4; ++b)
+          tma_load_2d(dst + b * kBoxBytes, &wmap, kc * kKC, box_row(g, tile, b), &k.full[slot], pol);
+        return true;
+      };
+      const int npre = n < NS ? n : NS;
+      bool ok = true;
+      for (int i = 0; i < npre && ok; ++i) ok = issue_w(i);
+      pdl_wait();
+      const int K = g.K;
+      for (int i = 0; i < n && ok; ++i) {
+        if (i >= npre) ok = issue_w(i);
+        if (!ok) break;
+        const int slot = i % NS;
+        const int kc = (u_begin + i) % g.nks;
+        unsigned char* xdst = smem + S::xs + (size_t)slot * S::XS;
+        const int cols = min(kKC, K - kc * kKC);
+        const uint32_t gbytes = NORM ? (uint32_t)cols * 2u : 0u;
+        mbar_arrive_expect_tx(&k.xfull[slot], (uint32_t)S::XB + gbytes);
+        tma_load_2d(xdst, &xmap, kc * kKC, 0, &k.xfull[slot], pol);
+        if (NORM) bulk_g2s(xdst + S::XB, a.gnorm + (size_t)kc * kKC, gbytes, &k.xfull[slot], pol);
+      }
+      if (!ok) flag_timeout(a.B);
+      // every copy has landed before the block exits
+      for (int j = n > NS ? n - NS : 0; j < n; ++j) {
+        mbar_wait(&k.full[j % NS], (uint32_t)(j / NS) & 1u);
+        mbar_wait(&k.xfull[j % NS], (uint32_t)(j / NS) & 1u);
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    // ---------------- MMA issue (one thread)
+    if (lane == 0 && n > 0) {
+      int tc = -1;
+      if (!mma_units(k, g, u_begin, n, 0, tc, tmem)) flag_timeout(a.B);
+      // every MMA has completed before TMEM is released
+      tc_commit(k.drain);
+      if (!mbar_wait(k.drain, 0)) flag_timeout(a.B);
+    }
+  } else {
+    // ---------------- workers: operand tiles and epilogues
+    pdl_wait();
+    int pos0, M;
+    resolve_rows(a.B.ctl, a.sel, pos0, M);
+    if (M > TP) M = TP;  // the launcher picks TP >= M
+    k.clear_operands(tid);
+    int tc = -1;
+    bool ok = true;
+    worker_units<TP, KIND, NORM>(a, k, tmem, u_begin, n, 0, tc, ok, pos0, M);
 
     // ---- exit head: per-block statistics, and the last block's fixed-order merge
     if constexpr (KIND == kKHead) {
+      HeadPart* run = k.run;
+      HeadPart* comb = k.comb;
+      int* sflag = k.sflag;
       HeadPart* sl = static_cast<HeadPart*>(a.B.head_part);
       named_sync(1, kWThreads);
       if (tid < M) {
@@ -739,6 +800,189 @@ __global__ void __launch_bounds__(kTThreads, 1)
   }
 
   // TMEM is released once every MMA has completed and every read is done
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == kMmaWarp) tc_dealloc(tmem, S::kCols);
+}
+
+// ---------------------------------------------------------- the chain kernel
+//
+// One layer's MLP half and the next layer's QKV in one persistent launch:
+// phase 0 O projection + residual, 1 RMSNorm + gate/up + SwiGLU, 2 down
+// projection + residual, 3 (optional) RMSNorm + QKV + RoPE + KV append of the
+// next layer.  Each phase is exactly the matrix pass of k_tile (same units,
+// same stream-K split, same arithmetic and fix-up order, so results are bit
+// for bit those of four k_tile launches).  What changes is the pipeline: a
+// weight thread streams every phase's units through the ring without
+// waiting for anything but free slots, so the next phase's weights arrive
+// while the current phase finishes its split tiles; an input thread issues a
+// phase's input slices once every block has finished the previous phase (a
+// grid-wide arrival counter; the grid is one block per SM, all resident).
+
+constexpr int kXWarp = kWorkers + 2;
+constexpr int kCThreads = (kWorkers + 3) * 32;
+
+struct ChainArgs {
+  TArgs ph[4];
+  int nph;
+  uint32_t* bar;  // [0] arrivals of finished phases, [1] blocks done (self-resetting)
+};
+
+struct ChainMaps {
+  CUtensorMap w[4];  // weights of each phase
+  CUtensorMap x[4];  // input rows of each phase
+};
+
+// Waits until *bar >= target (acquire); false after ~2^24 polls.
+__device__ __forceinline__ bool grid_wait(const uint32_t* bar, uint32_t target) {
+  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(bar) : "memory");
+    if (v >= target) return true;
+    __nanosleep(32);
+  }
+  return false;
+}
+
+template <int TP, bool QKV4>
+__global__ void __launch_bounds__(kCThreads, 1)
+    k_chain(const __grid_constant__ ChainMaps maps, const __grid_constant__ ChainArgs ca) {
+  using S = TL<TP, false>;
+  constexpr int NS = S::NS;
+  constexpr int NPH = QKV4 ? 4 : 3;
+  extern __shared__ unsigned char smem_raw[];
+  Blk<TP, false> k(smem_raw);
+  unsigned char* smem = k.smem;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
+  const int P = ca.ph[0].g.P;
+  const uint32_t tmem = k.setup(warp, kMmaWarp);
+  pdl_launch_dependents();
+
+  if (warp == kTmaWarp) {
+    // ---------------- weights: every phase, back to back
+    if (lane == 0) {
+      const uint64_t pol = evict_first_policy();
+      for (int p = 0; p < NPH; ++p) tma_prefetch_desc(&maps.w[p]);
+      bool ok = true;
+      int gi = 0;
+      for (int p = 0; p < NPH && ok; ++p) {
+        const TGeom& g = ca.ph[p].g;
+        const int u_begin = t_start(g, blockIdx.x), n = t_start(g, blockIdx.x + 1) - u_begin;
+        for (int i = 0; i < n; ++i, ++gi) {
+          const int slot = gi % NS;
+          if (!mbar_wait(&k.empty[slot], ((uint32_t)(gi / NS) & 1u) ^ 1u)) {
+            ok = false;
+            break;
+          }
+          const int u = u_begin + i;
+          const int tile = u / g.nks, kc = u - tile * g.nks;
+          mbar_arrive_expect_tx(&k.full[slot], (uint32_t)kWBytes);
+          unsigned char* dst = smem + S::ring + (size_t)slot * kWBytes;
+#pragma unroll
+          for (int b = 0; b < 4; ++b)
+            tma_load_2d(dst + b * kBoxBytes, &maps.w[p], kc * kKC, box_row(g, tile, b), &k.full[slot],
+                        pol);
+        }
+      }
+      if (!ok) flag_timeout(ca.ph[0].B);
+      for (int j = gi > NS ? gi - NS : 0; j < gi; ++j) mbar_wait(&k.full[j % NS], (uint32_t)(j / NS) & 1u);
+    }
+  } else if (warp == kXWarp) {
+    // ---------------- input slices: phase p after every block finished p - 1
+    if (lane == 0) {
+      const uint64_t pol = evict_first_policy();
+      for (int p = 0; p < NPH; ++p) tma_prefetch_desc(&maps.x[p]);
+      pdl_wait();
+      bool ok = true;
+      int gi = 0;
+      for (int p = 0; p < NPH; ++p) {
+        const TArgs& a = ca.ph[p];
+        const TGeom& g = a.g;
+        if (p > 0) {
+          if (!grid_wait(ca.bar, (uint32_t)(p * P))) ok = false;
+          // inputs written by other blocks' generic stores, read by TMA
+          asm volatile("fence.proxy.async.global;" ::: "memory");
+        }
+        const int u_begin = t_start(g, blockIdx.x), n = t_start(g, blockIdx.x + 1) - u_begin;
+        const bool norm = a.gnorm != nullptr;
+        for (int i = 0; i < n && ok; ++i, ++gi) {
+          const int slot = gi % NS;
+          if (!mbar_wait(&k.empty[slot], ((uint32_t)(gi / NS) & 1u) ^ 1u)) {
+            ok = false;
+            break;
+          }
+          const int kc = (u_begin + i) % g.nks;
+          unsigned char* xdst = smem + S::xs + (size_t)slot * S::XS;
+          const int cols = min(kKC, g.K - kc * kKC);
+          const uint32_t gbytes = norm ? (uint32_t)cols * 2u : 0u;
+          mbar_arrive_expect_tx(&k.xfull[slot], (uint32_t)S::XB + gbytes);
+          tma_load_2d(xdst, &maps.x[p], kc * kKC, 0, &k.xfull[slot], pol);
+          if (norm) bulk_g2s(xdst + S::XB, a.gnorm + (size_t)kc * kKC, gbytes, &k.xfull[slot], pol);
+        }
+        if (!ok) break;
+      }
+      if (!ok) flag_timeout(ca.ph[0].B);
+      for (int j = gi > NS ? gi - NS : 0; j < gi; ++j) mbar_wait(&k.xfull[j % NS], (uint32_t)(j / NS) & 1u);
+    }
+  } else if (warp == kMmaWarp) {
+    // ---------------- MMA issue (one thread), every phase
+    if (lane == 0) {
+      int tc = -1, gi = 0;
+      bool ok = true;
+      for (int p = 0; p < NPH && ok; ++p) {
+        const TGeom& g = ca.ph[p].g;
+        const int u_begin = t_start(g, blockIdx.x), n = t_start(g, blockIdx.x + 1) - u_begin;
+        ok = mma_units(k, g, u_begin, n, gi, tc, tmem);
+        gi += n;
+      }
+      if (!ok) flag_timeout(ca.ph[0].B);
+      tc_commit(k.drain);
+      if (!mbar_wait(k.drain, 0)) flag_timeout(ca.ph[0].B);
+    }
+  } else if (warp < kWorkers) {
+    // ---------------- workers, phase by phase
+    pdl_wait();
+    int pos0, M;
+    resolve_rows(ca.ph[0].B.ctl, ca.ph[0].sel, pos0, M);
+    if (M > TP) M = TP;
+    k.clear_operands(tid);
+    int tc = -1, gi = 0;
+    bool ok = true;
+    auto phase = [&](auto kind, auto norm, int p) {
+      constexpr int KIND = decltype(kind)::value;
+      constexpr bool NORM = decltype(norm)::value;
+      const TArgs& a = ca.ph[p];
+      if (p > 0) {
+        // every block finished phase p - 1: one thread acquires, the CTA
+        // barrier orders the other workers' reads after it (all reads of
+        // other blocks' outputs go to L2)
+        if (tid == 0) *k.sflag = grid_wait(ca.bar, (uint32_t)(p * P)) ? 1 : 0;
+        named_sync(1, kWThreads);
+        if (!*k.sflag) ok = false;
+        named_sync(1, kWThreads);
+      }
+      const int u_begin = t_start(a.g, blockIdx.x), n = t_start(a.g, blockIdx.x + 1) - u_begin;
+      worker_units<TP, KIND, NORM>(a, k, tmem, u_begin, n, gi, tc, ok, pos0, M);
+      gi += n;
+      // this block's outputs of phase p are written: arrive
+      __threadfence();
+      named_sync(1, kWThreads);
+      if (tid == 0) atomicAdd(ca.bar, 1u);
+    };
+    phase(std::integral_constant<int, kKResid>{}, std::false_type{}, 0);
+    phase(std::integral_constant<int, kKGateUp>{}, std::true_type{}, 1);
+    phase(std::integral_constant<int, kKResid>{}, std::false_type{}, 2);
+    if constexpr (QKV4) phase(std::integral_constant<int, kKQKV>{}, std::true_type{}, 3);
+    // the last block out resets the counters for the next launch (every
+    // block has passed all of its waits by now)
+    if (tid == 0 && atomicAdd(ca.bar + 1, 1u) == (uint32_t)(P - 1)) {
+      ca.bar[0] = 0u;
+      ca.bar[1] = 0u;
+      __threadfence();
+    }
+  }
+
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -808,6 +1052,21 @@ cudaError_t prep_one() {
                               (int)TL<TP, KIND == kKHead>::total);
 }
 
+template <int TP, bool QKV4>
+cudaError_t chain_launch(const ChainMaps& m, const ChainArgs& a, cudaStream_t st) {
+  return launch_ex(k_chain<TP, QKV4>, dim3(a.ph[0].g.P), dim3(kCThreads), TL<TP, false>::total, st,
+                   m, a);
+}
+
+template <int TP>
+cudaError_t prep_chain() {
+  cudaError_t e = cudaFuncSetAttribute(k_chain<TP, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)TL<TP, false>::total);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(k_chain<TP, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)TL<TP, false>::total);
+}
+
 template <int KIND, bool NORM>
 cudaError_t prep_kind() {
   cudaError_t e = prep_one<8, KIND, NORM>();
@@ -848,6 +1107,9 @@ cudaError_t prepare_tile_kernels() {
   if ((e = prep_kind<kKQKV, true>()) != cudaSuccess) return e;
   if ((e = prep_kind<kKGateUp, true>()) != cudaSuccess) return e;
   if ((e = prep_kind<kKResid, false>()) != cudaSuccess) return e;
+  if ((e = prep_chain<8>()) != cudaSuccess) return e;
+  if ((e = prep_chain<16>()) != cudaSuccess) return e;
+  if ((e = prep_chain<24>()) != cudaSuccess) return e;
   return prep_kind<kKHead, true>();
 }
 
@@ -888,6 +1150,57 @@ cudaError_t launch_tile_part(const Dims& D, const Bufs& B, const TileMaps& tm, c
       return tile_dispatch<kKResid, false>(*w.tm[3], tm.act, a, mrows, st);
     default:
       return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_tile_chain(const Dims& D, const Bufs& B, const TileMaps& tm, const LayerW& w,
+                              const LayerW* next, int layer, RowSel sel, int mrows,
+                              cudaStream_t st) {
+  const int tp = tp_index(mrows);
+  ChainArgs ca{};
+  ChainMaps cm{};
+  for (int p = 0; p < 4; ++p) {
+    ca.ph[p].D = D;
+    ca.ph[p].B = B;
+    ca.ph[p].sel = sel;
+    ca.ph[p].layer = layer;
+    ca.ph[p].ss_in = -1;
+  }
+  // O projection + residual
+  ca.ph[0].g = make_tgeom(D, D.d, D.qd, kTMapLinear);
+  ca.ph[0].which = 1;
+  cm.w[0] = *w.tm[1];
+  cm.x[0] = tm.attn_out[tp];
+  // RMSNorm + gate/up + SwiGLU
+  ca.ph[1].g = make_tgeom(D, 2 * D.F, D.d, kTMapGateUp);
+  ca.ph[1].gnorm = static_cast<const __nv_bfloat16*>(w.ffn_norm);
+  ca.ph[1].ss_in = 1;
+  cm.w[1] = *w.tm[2];
+  cm.x[1] = tm.h[tp];
+  // down projection + residual
+  ca.ph[2].g = make_tgeom(D, D.d, D.F, kTMapLinear);
+  ca.ph[2].which = 0;
+  cm.w[2] = *w.tm[3];
+  cm.x[2] = tm.act[tp];
+  ca.nph = 3;
+  if (next) {  // the next layer's RMSNorm + QKV + RoPE + KV append
+    ca.ph[3].g = make_tgeom(D, (D.Hq + 2 * D.Hkv) * D.hd, D.d, kTMapQKV);
+    ca.ph[3].gnorm = static_cast<const __nv_bfloat16*>(next->attn_norm);
+    ca.ph[3].ss_in = 0;
+    ca.ph[3].layer = layer + 1;
+    cm.w[3] = *next->tm[0];
+    cm.x[3] = tm.h[tp];
+    ca.nph = 4;
+  }
+  for (int p = 0; p < ca.nph; ++p)
+    if (ca.ph[p].g.T < 1 || ca.ph[p].g.T > (1 << 22) || ca.ph[p].g.P < 1 ||
+        ca.ph[p].g.P > kMaxBlocksDev)
+      return cudaErrorInvalidValue;
+  ca.bar = B.chain_bar;
+  switch (tp) {
+    case 0: return next ? chain_launch<8, true>(cm, ca, st) : chain_launch<8, false>(cm, ca, st);
+    case 1: return next ? chain_launch<16, true>(cm, ca, st) : chain_launch<16, false>(cm, ca, st);
+    default: return next ? chain_launch<24, true>(cm, ca, st) : chain_launch<24, false>(cm, ca, st);
   }
 }
 

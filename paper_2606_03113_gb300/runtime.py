@@ -188,16 +188,28 @@ class Engine:
             pass
 
 
-def kernels_per_round(trace: dict, n_layers: int, kind: int) -> int:
+def pass_launches(n_layers: int, bf16: bool = True) -> int:
+    """Kernel launches of a pass over n layers: bf16 runs the first QKV, then
+    per layer attention and one chained launch (O, gate/up, down, next QKV);
+    fp32 launches the five layer kernels per layer."""
+    if n_layers <= 0:
+        return 0
+    return 2 * n_layers + 1 if bf16 else S.KERNELS_PER_LAYER * n_layers
+
+
+def kernels_per_round(trace: dict, n_layers: int, kind: int, bf16: bool = True) -> int:
     """Kernel launches of one round of the round graph, from its record:
-    round_begin, walk (embed, 5 per layer, head, decide per visited segment),
-    draft_begin, drafts (embed, 5 per layer, head, decide), verify (embed,
-    5 per layer, head), accept."""
-    per_layer = S.KERNELS_PER_LAYER
+    round_begin, walk (embed; per visited segment its layers, head, decide),
+    draft_begin, drafts (embed, layers 1..l*, head, decide), verify (embed,
+    all layers, head), accept."""
     n = 1  # round_begin
     if trace["kcap"] > 0:
-        n += 1 + trace["lstar"] * per_layer + 2 * len(trace["visited"])
+        prev = 0
+        n += 1  # embed
+        for c in trace["visited"]:
+            n += pass_launches(c - prev, bf16) + 2
+            prev = c
         n += 1  # draft_begin
-        n += (trace["k"] - 1) * (1 + trace["lstar"] * per_layer + 2)
-    n += 1 + n_layers * per_layer + 1 + 1
+        n += (trace["k"] - 1) * (1 + pass_launches(trace["lstar"], bf16) + 2)
+    n += 1 + pass_launches(n_layers, bf16) + 1 + 1
     return n

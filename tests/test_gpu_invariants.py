@@ -119,3 +119,43 @@ def test_error_paths_return_status():
     toks, _, _ = eng.generate(4)
     assert len(toks) == 4
     eng.close()
+
+
+def test_chained_layer_launch_equals_one_launch_per_matrix():
+    """The persistent launch that runs a layer's O, gate/up and down and the
+    next layer's QKV as phases computes exactly what one launch per matrix
+    computes: teacher-forced logits and statistics at every exit depth are
+    equal bit for bit, for one row and for a verification tile."""
+    import os
+    from paper_2606_03113_gb300.runtime import Engine
+    w, dm, eng_chain, om = setup("7b")
+    ids = prompt(w)
+    n0 = len(ids) - 13
+    old = os.environ.get("SSD_NO_CHAIN")
+    os.environ["SSD_NO_CHAIN"] = "1"
+    try:
+        eng_plain = Engine(dm, w.max_seq)
+        outs = {}
+        for name, e in (("plain", eng_plain), ("chain", None)):
+            if e is None:
+                os.environ["SSD_NO_CHAIN"] = "0"
+                e = Engine(dm, w.max_seq)  # re-reads the switch
+            e.set_ar()
+            e.prefill(ids[:n0])
+            res = []
+            for l_exit in (1, w.shape.n_layers // 2, w.shape.n_layers):
+                for M in (1, 13):
+                    z, st = e.forward_exit(ids[n0:n0 + M], n0, l_exit)
+                    res.append((z, [s["argmax"] for s in st], [s["entropy"] for s in st]))
+            e.prefill(ids)
+            toks, _, _ = e.generate(24)
+            outs[name] = (res, toks)
+            e.close()
+    finally:
+        if old is None:
+            os.environ.pop("SSD_NO_CHAIN", None)
+        else:
+            os.environ["SSD_NO_CHAIN"] = old
+    for (za, aa, ea), (zb, ab, eb) in zip(outs["plain"][0], outs["chain"][0]):
+        assert np.array_equal(za, zb) and aa == ab and ea == eb
+    assert np.array_equal(outs["plain"][1], outs["chain"][1])
