@@ -277,6 +277,18 @@ __device__ __forceinline__ void t_head_token(const TArgs& a, int tile, int s, in
 
 // ------------------------------------------------------------ the kernels
 
+// Waits until *bar >= target (acquire load); false after ~2^24 polls.
+__device__ __forceinline__ bool counter_wait(const uint32_t* bar, uint32_t target) {
+  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(bar) : "memory");
+    if (v >= target) return true;
+    __nanosleep(32);
+  }
+  return false;
+}
+
+
 // Shared-memory views of one block (layout TL<TP, HEAD>).
 template <int TP, bool HEAD>
 struct Blk {
@@ -488,28 +500,35 @@ __device__ void worker_units(const TArgs& a, const Blk<TP, KIND == kKHead>& k, u
       if constexpr (KIND == kKResid) tile_ss(ssv, tile);
       return;
     }
-    // shared with neighbouring blocks: publish this block's partial sums
-    const int slot2 = tile == first_tile ? 0 : 1;
-    float* mine = a.B.gpart + ((size_t)blockIdx.x * 2 + slot2) * 2 * kMaxM * 128;
-#pragma unroll
-    for (int lt = 0; lt < LTN; ++lt) {
-      const int t = 2 * lt + grp;
-      if (t >= M) break;
-      mine[(size_t)t * 128 + srow] = grp ? v[0][2 * lt + 1] : v[0][2 * lt];
-      mine[(size_t)(kMaxM + t) * 128 + srow] = grp ? v[1][2 * lt + 1] : v[1][2 * lt];
-    }
-    __threadfence();
-    named_sync(1, kWThreads);
+    // Shared with neighbouring blocks.  The tile's first contributor b0 (for
+    // which it is always the last tile of its range) finishes it: the others
+    // publish their partial sums and count themselves in without waiting;
+    // b0 waits for that count, keeps its own partial in registers and adds
+    // the others' in block order.
     const int b0 = t_block_of(g, t0), b1 = t_block_of(g, t1 - 1);
+    if ((int)blockIdx.x != b0) {
+      const int slot2 = tile == first_tile ? 0 : 1;
+      float* mine = a.B.gpart + ((size_t)blockIdx.x * 2 + slot2) * 2 * kMaxM * 128;
+#pragma unroll
+      for (int lt = 0; lt < LTN; ++lt) {
+        const int t = 2 * lt + grp;
+        if (t >= M) break;
+        mine[(size_t)t * 128 + srow] = grp ? v[0][2 * lt + 1] : v[0][2 * lt];
+        mine[(size_t)(kMaxM + t) * 128 + srow] = grp ? v[1][2 * lt + 1] : v[1][2 * lt];
+      }
+      __threadfence();
+      named_sync(1, kWThreads);
+      if (tid == 0) atomicAdd(&a.B.tile_counter[tile], 1u);  // result unused: a reduction
+      return;
+    }
     if (tid == 0) {
       int contrib = 0;
       for (int b = b0; b <= b1; ++b) contrib += t_start(g, b) < t_start(g, b + 1);
-      *sflag = atomicAdd(&a.B.tile_counter[tile], 1u) == (unsigned)(contrib - 1);
+      *sflag = counter_wait(&a.B.tile_counter[tile], (uint32_t)(contrib - 1)) ? 1 : 0;
+      a.B.tile_counter[tile] = 0u;
     }
     named_sync(1, kWThreads);
-    if (!*sflag) return;
-    __threadfence();
-    if (tid == 0) a.B.tile_counter[tile] = 0u;
+    if (!*sflag && tid == 0) flag_timeout(a.B);
     float ss_sp[LTN];
 #pragma unroll
     for (int lt = 0; lt < LTN; ++lt) ss_sp[lt] = 0.f;
@@ -526,10 +545,14 @@ __device__ void worker_units(const TArgs& a, const Blk<TP, KIND == kKHead>& k, u
     constexpr int GB = LTN <= 4 ? 4 : (LTN <= 8 ? 2 : 1);
     float u0[LTN], u1[LTN];
 #pragma unroll
-    for (int lt = 0; lt < LTN; ++lt) u0[lt] = u1[lt] = 0.f;
+    for (int lt = 0; lt < LTN; ++lt) {  // b0's own partial first (0 + x: exactly x)
+      const int t = 2 * lt + grp;
+      u0[lt] = t < M ? (grp ? v[0][2 * lt + 1] : v[0][2 * lt]) : 0.f;
+      u1[lt] = t < M ? (grp ? v[1][2 * lt + 1] : v[1][2 * lt]) : 0.f;
+    }
     if (M == 1) {
       // one token (drafting, autoregressive steps): sixteen contributors per round
-      for (int b = grp == 0 ? b0 : b1 + 1; b <= b1; b += 16) {
+      for (int b = grp == 0 ? b0 + 1 : b1 + 1; b <= b1; b += 16) {
         float c0[16], c1[16];
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
@@ -554,7 +577,7 @@ __device__ void worker_units(const TArgs& a, const Blk<TP, KIND == kKHead>& k, u
         }
       }
     } else
-      for (int b = b0; b <= b1; b += GB) {
+      for (int b = b0 + 1; b <= b1; b += GB) {
         float c0[GB][LTN], c1[GB][LTN];
 #pragma unroll
         for (int j = 0; j < GB; ++j) {
@@ -834,17 +857,6 @@ struct ChainMaps {
   CUtensorMap x[4];  // input rows of each phase
 };
 
-// Waits until *bar >= target (acquire); false after ~2^24 polls.
-__device__ __forceinline__ bool grid_wait(const uint32_t* bar, uint32_t target) {
-  for (uint32_t i = 0; i < kSpinLimit; ++i) {
-    uint32_t v;
-    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(bar) : "memory");
-    if (v >= target) return true;
-    __nanosleep(32);
-  }
-  return false;
-}
-
 template <int TP, bool QKV4>
 __global__ void __launch_bounds__(kCThreads, 1)
     k_chain(const __grid_constant__ ChainMaps maps, const __grid_constant__ ChainArgs ca) {
@@ -900,7 +912,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
         const TArgs& a = ca.ph[p];
         const TGeom& g = a.g;
         if (p > 0) {
-          if (!grid_wait(ca.bar, (uint32_t)(p * P))) ok = false;
+          if (!counter_wait(ca.bar, (uint32_t)(p * P))) ok = false;
           // inputs written by other blocks' generic stores, read by TMA
           asm volatile("fence.proxy.async.global;" ::: "memory");
         }
@@ -957,7 +969,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
         // every block finished phase p - 1: one thread acquires, the CTA
         // barrier orders the other workers' reads after it (all reads of
         // other blocks' outputs go to L2)
-        if (tid == 0) *k.sflag = grid_wait(ca.bar, (uint32_t)(p * P)) ? 1 : 0;
+        if (tid == 0) *k.sflag = counter_wait(ca.bar, (uint32_t)(p * P)) ? 1 : 0;
         named_sync(1, kWThreads);
         if (!*k.sflag) ok = false;
         named_sync(1, kWThreads);
