@@ -251,6 +251,24 @@ __device__ __forceinline__ void t_pair(const TArgs& a, int tile, int s, int t, i
   }
 }
 
+// Residual add with the rows' previous values already loaded (split-tile
+// fix-ups load them together with the contributors' partial sums).
+__device__ __forceinline__ void t_resid_pre(const TArgs& a, int tile, int s, int t, float v0,
+                                            float v1, float h0, float h1, float& ss) {
+  const int r0 = trow(a.g, tile, s), r1 = trow(a.g, tile, s + 128);
+  float* hm = a.B.h + (size_t)t * a.D.d;
+  if (r0 >= 0) {
+    const float h = h0 + v0;
+    hm[r0] = h;
+    ss = fmaf(h, h, ss);
+  }
+  if (r1 >= 0) {
+    const float h = h1 + v1;
+    hm[r1] = h;
+    ss = fmaf(h, h, ss);
+  }
+}
+
 // Exit head, one token, whole warp: the logits of the lane's two rows enter
 // a per-lane partial, merged over the warp by a fixed shuffle tree; lane 0
 // merges the result into `acc` (shared memory, one slot per warp and token).
@@ -543,6 +561,18 @@ __device__ void worker_units(const TArgs& a, const Blk<TP, KIND == kKHead>& k, u
     // round trips rather than one per contributor and token.  Unused slots
     // read block 0's partials (valid memory) and add zero.
     constexpr int GB = LTN <= 4 ? 4 : (LTN <= 8 ? 2 : 1);
+    // residual kernels: the rows' previous values, loaded with the partials
+    float hp0[LTN], hp1[LTN];
+    if constexpr (KIND == kKResid) {
+      const int r0 = trow(g, tile, srow), r1 = trow(g, tile, srow + 128);
+#pragma unroll
+      for (int lt = 0; lt < LTN; ++lt) {
+        const int t = 2 * lt + grp;
+        const float* hm = a.B.h + (size_t)(t < M ? t : 0) * a.D.d;
+        hp0[lt] = (t < M && r0 >= 0) ? __ldcg(hm + r0) : 0.f;
+        hp1[lt] = (t < M && r1 >= 0) ? __ldcg(hm + r1) : 0.f;
+      }
+    }
     float u0[LTN], u1[LTN];
 #pragma unroll
     for (int lt = 0; lt < LTN; ++lt) {  // b0's own partial first (0 + x: exactly x)
@@ -614,6 +644,8 @@ __device__ void worker_units(const TArgs& a, const Blk<TP, KIND == kKHead>& k, u
       if (t >= M) break;
       if constexpr (KIND == kKHead)
         t_head_token(a, tile, srow, t, rs_t[lt], u0[lt], u1[lt], &spl[warp * kLT + lt], lane);
+      else if constexpr (KIND == kKResid)
+        t_resid_pre(a, tile, srow, t, u0[lt], u1[lt], hp0[lt], hp1[lt], ss_sp[lt]);
       else
         t_pair<KIND>(a, tile, srow, t, pos0, rs_t[lt], u0[lt], u1[lt], ss_sp[lt]);
     }
