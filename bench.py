@@ -38,6 +38,9 @@ CLOCK_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.a
                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
 
+SAMPLE_SEED = 7  # uniforms of the sampled-decoding comparison lines
+
+
 def measured_peaks() -> dict:
     p = os.path.join(REPO, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -386,13 +389,14 @@ def main():
                          updates=tlog.updates, collect_s=round(t1 - t0, 1),
                          train_s=round(t2 - t1, 1))
 
-    def set_policy(kind, l=0, k=0, q=None):
+    def set_policy(kind, l=0, k=0, q=None, temperature=0.0):
+        smp = dict(temperature=temperature, sample_seed=SAMPLE_SEED)
         if kind == "ar":
-            eng.set_ar()
+            eng.set_ar(**smp)
         elif kind == "static":
-            eng.set_static(l, k, kmax=w.kmax)
+            eng.set_static(l, k, kmax=w.kmax, **smp)
         else:
-            eng.set_lede(w, qp if q is None else q)
+            eng.set_lede(w, qp if q is None else q, **smp)
 
     L = w.shape.n_layers
     if args.kernels_only:
@@ -456,19 +460,25 @@ def main():
 
     compare = {}
     if not args.no_compare and args.policy == "lede":
-        runs = [("ar", "ar", (0, 0), None), ("static_layerskip", "static", static_lk, None),
-                ("static_l16_k4", "static", (L // 2, 4), None),
-                ("static_l24_k2", "static", (3 * L // 4, 2), None)]
+        runs = [("ar", "ar", (0, 0), None, 0.0),
+                ("static_layerskip", "static", static_lk, None, 0.0),
+                ("static_l16_k4", "static", (L // 2, 4), None, 0.0),
+                ("static_l24_k2", "static", (3 * L // 4, 2), None, 0.0)]
         if qnet_info["kind"] != "seeded":
-            runs.append(("lede_seeded_qnet", "lede", (0, 0), seeded_qp))
-        for name, kind, lk, q in runs:
-            set_policy(kind, *lk, q=q)
+            runs.append(("lede_seeded_qnet", "lede", (0, 0), seeded_qp, 0.0))
+        # sampled decoding at the paper's language-modelling temperature
+        runs += [("ar_sampled_t0.6", "ar", (0, 0), None, 0.6),
+                 ("lede_sampled_t0.6", "lede", (0, 0), None, 0.6)]
+        for name, kind, lk, q, temp in runs:
+            set_policy(kind, *lk, q=q, temperature=temp)
             time_generate(eng, ids, n_new, barrier)
             r = time_generate(eng, ids, n_new, barrier)
             tr = r[2]
             compare[name] = dict(tok_s=r[1] / (r[0] / 1e3), l=lk[0], k=lk[1],
                                  acc_rate=sum(t["a"] for t in tr) / max(1, sum(t["k"] for t in tr)),
                                  gb_per_token=sum(round_bytes(w, t) for t in tr) / r[1] / 1e9)
+            if temp > 0:
+                compare[name]["temperature"] = temp
         ar_bytes = L * w.shape.layer_weight_bytes() + w.shape.lm_head_bytes()
         compare["ar_roofline_tok_s"] = peak * 1e9 / ar_bytes
 

@@ -114,6 +114,13 @@ typedef struct {
   int32_t topk;    /* k of the token confidence, 1..8 (paper: 5) */
   int32_t fixed_k; /* LEDE: 0 = adaptive drafting; 1..16 = fixed draft length */
   float conf_threshold; /* THRESHOLD: (0, 1] */
+  /* Sampled decoding (speculative sampling, §4.1): temperature 0 is greedy;
+   * > 0 samples drafts from the exit distribution and the emitted tokens
+   * from the full model's, both at this temperature, with the acceptance
+   * rule that keeps the full model's distribution; uniforms come from the
+   * counter-based generator keyed by sample_seed and the round's position. */
+  float temperature;
+  uint32_t sample_seed;
 } ssd_policy;
 
 typedef struct {
@@ -136,11 +143,19 @@ typedef struct {
   int32_t verify_tok[SSD_TRACE_MAXK + 1];
   int32_t emitted[SSD_TRACE_MAXK + 1];
   int32_t q_action[SSD_TRACE_MAXQ];
-  float draft_margin[SSD_TRACE_MAXK];      /* top-1 minus top-2 logit of each draft */
+  float draft_margin[SSD_TRACE_MAXK];      /* top-1 minus top-2 logit of each draft (greedy);
+                                            * sampled: distance of the draw to the nearer end
+                                            * of the token's CDF interval, over the mass */
   float verify_margin[SSD_TRACE_MAXK + 1];
   float verify_pmax[SSD_TRACE_MAXK + 1];
   float q_val[SSD_TRACE_MAXQ][2];
   float q_state[SSD_TRACE_MAXQ][3];
+  /* sampled decoding only: margin of each acceptance test of d_i,
+   * (p(d) - r q(d)) / max(p(d), r q(d)) (> 0 keeps d_i), and the margin of
+   * the round's last draw (as draft_margin) */
+  int32_t sampled, pad2;
+  float accept_margin[SSD_TRACE_MAXK];
+  float fix_margin;
 } ssd_round_trace;
 
 typedef struct ssd_ctx ssd_ctx;
@@ -161,8 +176,10 @@ ssd_status ssd_set_policy(ssd_ctx* ctx, const ssd_policy* policy);
 
 /* Runs ids[0..n) (host) through the full model from position 0, seeds the
  * C_trace window with the full model's max-probabilities of the last trace_T
- * positions, and returns the greedy next token, which becomes the pending
- * token.  Needs n + 1 <= max_seq.  Synchronises the stream once. */
+ * positions, and returns the next token, which becomes the pending token:
+ * the greedy one, or with a policy temperature > 0 (set before this call) a
+ * draw from the full model's distribution at that temperature, its uniform
+ * keyed by (sample_seed, n - 1).  Needs n + 1 <= max_seq.  Synchronises the stream once. */
 ssd_status ssd_prefill(ssd_ctx* ctx, const int32_t* ids, int32_t n, int32_t* first_token);
 
 /* Like ssd_prefill over ids[0..n-1) but takes ids[n-1] as the pending token

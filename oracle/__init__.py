@@ -44,7 +44,8 @@ class Policy(C.Structure):
                 ("kmax", C.c_int32), ("static_l", C.c_int32), ("static_k", C.c_int32),
                 ("q_in", C.c_int32), ("q_hidden", C.c_int32), ("trace_T", C.c_int32),
                 ("topk", C.c_int32), ("q_params", C.c_void_p), ("fixed_k", C.c_int32),
-                ("conf_threshold", C.c_double)]
+                ("conf_threshold", C.c_double), ("temperature", C.c_double),
+                ("sample_seed", C.c_uint32)]
 
 
 class RoundLog(C.Structure):
@@ -55,7 +56,8 @@ class RoundLog(C.Structure):
                 ("emitted", C.c_int32 * (MAX_K + 1)), ("q_action", C.c_int32 * MAX_Q),
                 ("draft_margin", C.c_double * MAX_K), ("verify_margin", C.c_double * (MAX_K + 1)),
                 ("verify_pmax", C.c_double * (MAX_K + 1)), ("q_val", (C.c_double * 2) * MAX_Q),
-                ("q_state", (C.c_double * 3) * MAX_Q)]
+                ("q_state", (C.c_double * 3) * MAX_Q), ("sampled", C.c_int32),
+                ("accept_margin", C.c_double * MAX_K), ("fix_margin", C.c_double)]
 
     def as_dict(self) -> dict:
         k, a, n = self.k, self.a, self.n_emit
@@ -68,7 +70,9 @@ class RoundLog(C.Structure):
                     verify_pmax=list(self.verify_pmax[:k + 1]),
                     q_action=list(self.q_action[:nq]),
                     q_val=[tuple(self.q_val[i]) for i in range(nq)],
-                    q_state=[tuple(self.q_state[i]) for i in range(nq)])
+                    q_state=[tuple(self.q_state[i]) for i in range(nq)],
+                    sampled=bool(self.sampled), accept_margin=list(self.accept_margin[:k]),
+                    fix_margin=self.fix_margin)
 
 
 _lock = threading.Lock()
@@ -128,6 +132,11 @@ def lib():
             L.orc_trace_push.restype = None
             L.orc_prefill.argtypes = [p, p, i32, i32, p]
             L.orc_resume.argtypes = [p, p, i32, i32]
+            L.orc_prefill_sampled.argtypes = [p, p, i32, i32, C.c_double, C.c_uint32, p, p]
+            L.orc_tempered.argtypes = [p, i32, C.c_double, p]
+            L.orc_tempered.restype = None
+            L.orc_draw.argtypes = [p, i32, C.c_double, p]
+            L.orc_spec_step.argtypes = [p, p, i32, i32, C.c_double, C.c_double, p, p, p, p]
             L.orc_round.argtypes = [p, C.POINTER(Policy), i32, C.POINTER(RoundLog)]
             L.orc_generate.argtypes = [p, C.POINTER(Policy), i32, p, p, i32, p]
             L.orc_num_threads.argtypes = []
@@ -173,7 +182,8 @@ def qnet(params: np.ndarray, hidden: int, s) -> np.ndarray:
 
 def make_policy(kind: int, cand=(), kmax: int = 0, static_l: int = 0, static_k: int = 0,
                 q_params: np.ndarray | None = None, q_hidden: int = 0, trace_T: int = 20,
-                topk: int = 5, fixed_k: int = 0, conf_threshold: float = 0.0) -> Policy:
+                topk: int = 5, fixed_k: int = 0, conf_threshold: float = 0.0,
+                temperature: float = 0.0, sample_seed: int = 0) -> Policy:
     P = Policy()
     P.kind = kind
     P.n_cand = len(cand)
@@ -182,6 +192,7 @@ def make_policy(kind: int, cand=(), kmax: int = 0, static_l: int = 0, static_k: 
     P.kmax, P.static_l, P.static_k = kmax, static_l, static_k
     P.q_in, P.q_hidden, P.trace_T, P.topk = 3, q_hidden, trace_T, topk
     P.fixed_k, P.conf_threshold = fixed_k, conf_threshold
+    P.temperature, P.sample_seed = temperature, sample_seed
     if q_params is not None:
         arr = np.ascontiguousarray(q_params, dtype=np.float32)
         P._keep = arr  # keep alive
@@ -294,10 +305,16 @@ class Session:
     def trace_push(self, p: float):
         lib().orc_trace_push(self.h, p)
 
-    def prefill(self, ids, trace_T: int = 20) -> int:
+    def prefill(self, ids, trace_T: int = 20, temperature: float = 0.0, seed: int = 0) -> int:
+        """Prompt prefill; the first token is greedy, or drawn at `temperature`
+        (> 0) with the uniform keyed by (seed, n - 1); its draw margin is
+        left in `self.prefill_margin`."""
         ids = np.ascontiguousarray(ids, dtype=np.int32)
         first = np.zeros(1, dtype=np.int32)
-        _check(lib().orc_prefill(self.h, _ptr(ids), ids.size, trace_T, _ptr(first)), "orc_prefill")
+        mg = np.zeros(1, dtype=np.float64)
+        _check(lib().orc_prefill_sampled(self.h, _ptr(ids), ids.size, trace_T, temperature, seed,
+                                         _ptr(first), _ptr(mg)), "orc_prefill")
+        self.prefill_margin = float(mg[0])
         return int(first[0])
 
     def resume(self, ids, trace_T: int = 20):
@@ -324,6 +341,36 @@ def matvec_synth(seed: int, tid: int, sigma: float, bf16: bool, row0: int, nrows
     _check(lib().orc_matvec_synth(seed, tid, sigma, 1 if bf16 else 0, row0, nrows, x.size, _ptr(x),
                                   _ptr(y)), "orc_matvec_synth")
     return y
+
+
+def tempered(z, temperature: float) -> np.ndarray:
+    """softmax(z / temperature) (orc_tempered)."""
+    z = np.ascontiguousarray(z, dtype=np.float64)
+    p = np.zeros_like(z)
+    lib().orc_tempered(_ptr(z), z.size, temperature, _ptr(p))
+    return p
+
+
+def draw(w, u: float):
+    """Inverse-CDF draw of orc_draw: (token, margin); token -1 when w has no mass."""
+    w = np.ascontiguousarray(w, dtype=np.float64)
+    mg = np.zeros(1, dtype=np.float64)
+    t = lib().orc_draw(_ptr(w), w.size, u, _ptr(mg))
+    return int(t), float(mg[0])
+
+
+def spec_step(p, q, d: int, r: float, u: float):
+    """One speculative-sampling acceptance test (orc_spec_step):
+    (emitted token, kept, accept margin, draw margin)."""
+    p = np.ascontiguousarray(p, dtype=np.float64)
+    q = np.ascontiguousarray(q, dtype=np.float64)
+    res = np.zeros_like(p)
+    kept = np.zeros(1, dtype=np.int32)
+    am = np.zeros(1, dtype=np.float64)
+    dm = np.zeros(1, dtype=np.float64)
+    t = lib().orc_spec_step(_ptr(p), _ptr(q), p.size, d, r, u, _ptr(res), _ptr(kept), _ptr(am),
+                            _ptr(dm))
+    return int(t), bool(kept[0]), float(am[0]), float(dm[0])
 
 
 def num_threads() -> int:

@@ -574,6 +574,76 @@ static int threshold_decide(const orc_policy* P, const orc_stats* st, orc_round_
   return a;
 }
 
+/* ------------------------------------------------------ sampled decoding */
+
+/* Tempered distribution of logits z at temperature T > 0:
+ * P(v) = exp((z_v - max z) / T) / sum_w exp((z_w - max z) / T). */
+void orc_tempered(const double* z, int V, double temperature, double* p) {
+  double zmax = z[0];
+  for (int v = 1; v < V; ++v)
+    if (z[v] > zmax) zmax = z[v];
+  double S = 0.0;
+  for (int v = 0; v < V; ++v) {
+    p[v] = exp((z[v] - zmax) / temperature);
+    S += p[v];
+  }
+  for (int v = 0; v < V; ++v) p[v] /= S;
+}
+
+/* Inverse-CDF draw from non-negative weights w (normalised or not): with
+ * W = sum_v w_v and C_v = w_0 + ... + w_v in token order, the token is the
+ * first v with C_v > u W.  *margin = min(u W - C_{v-1}, C_v - u W) / W, the
+ * distance of u W to the nearer end of the token's interval, relative to W.
+ * Returns -1 when W is not positive; when rounding leaves u W at or beyond
+ * the accumulated sum, the last token of positive weight (margin 0). */
+int orc_draw(const double* w, int V, double u, double* margin) {
+  double W = 0.0;
+  for (int v = 0; v < V; ++v) W += w[v];
+  *margin = 0.0;
+  if (!(W > 0.0)) return -1;
+  const double T = u * W;
+  double c = 0.0;
+  int last = -1;
+  for (int v = 0; v < V; ++v) {
+    const double nx = c + w[v];
+    if (w[v] > 0.0) last = v;
+    if (nx > T) {
+      *margin = fmin(T - c, nx - T) / W;
+      return v;
+    }
+    c = nx;
+  }
+  return last;
+}
+
+/* One acceptance test of speculative sampling (the acceptance rule of §4.1):
+ * draft d, drawn from the draft distribution q, is kept when r q(d) < p(d),
+ * i.e. with probability min(1, p(d) / q(d)); otherwise the emitted token is
+ * drawn with u from the residual max(0, p - q), normalised (from p itself
+ * should the residual carry no mass).  Either way the emitted token follows
+ * p.  res (V doubles) is scratch.  *accept_margin = (p(d) - r q(d)) /
+ * max(p(d), r q(d)), positive exactly when d is kept. */
+int orc_spec_step(const double* p, const double* q, int V, int d, double r, double u,
+                  double* res, int* accepted, double* accept_margin, double* draw_margin) {
+  const double pd = p[d], rq = r * q[d];
+  const double den = fmax(pd, rq);
+  *accept_margin = den > 0.0 ? (pd - rq) / den : 0.0;
+  *draw_margin = 0.0;
+  if (rq < pd) {
+    *accepted = 1;
+    return d;
+  }
+  *accepted = 0;
+  for (int v = 0; v < V; ++v) res[v] = fmax(p[v] - q[v], 0.0);
+  int t = orc_draw(res, V, u, draw_margin);
+  if (t < 0) t = orc_draw(p, V, u, draw_margin);
+  return t;
+}
+
+static double uniform_of(uint32_t seed, int pos, int purpose, int i) {
+  return (double)synth_sample_uniform(seed, (uint32_t)pos, (uint32_t)purpose, (uint32_t)i);
+}
+
 /* ------------------------------------------------------------ generation */
 
 static int check_policy(const orc_model* m, const orc_policy* P) {
@@ -603,7 +673,8 @@ static int check_policy(const orc_model* m, const orc_policy* P) {
 
 /* Full-model rows [0, n) of ids at positions 0..n-1; the max-probabilities of
  * the last min(T, n) rows seed the trace. */
-static int run_prompt(orc_sess* s, const int32_t* ids, int n, int trace_T, int32_t* last_argmax) {
+static int run_prompt(orc_sess* s, const int32_t* ids, int n, int trace_T, int32_t* last_argmax,
+                      double* z_last) {
   const orc_cfg* c = &s->m->c;
   int d = c->d_model;
   double* h = (double*)malloc(sizeof(double) * (size_t)n * d);
@@ -613,7 +684,7 @@ static int run_prompt(orc_sess* s, const int32_t* ids, int n, int trace_T, int32
   int first = n - trace_T > 0 ? n - trace_T : 0;
   for (int r = first; rc == ORC_OK && r < n; ++r) {
     orc_stats st;
-    rc = orc_exit_head(s->m, h + (int64_t)r * d, NULL, 1, &st);
+    rc = orc_exit_head(s->m, h + (int64_t)r * d, r == n - 1 ? z_last : NULL, 1, &st);
     orc_trace_push(s, st.pmax);
     if (r == n - 1 && last_argmax) *last_argmax = st.argmax;
   }
@@ -629,13 +700,44 @@ int orc_prefill(orc_sess* s, const int32_t* ids, int n, int trace_T, int32_t* fi
   s->kv_len = 0;
   s->have_x = 0;
   int32_t x = -1;
-  int rc = run_prompt(s, ids, n, trace_T, &x);
+  int rc = run_prompt(s, ids, n, trace_T, &x, NULL);
   if (rc) return rc;
   s->kv_len = n;
   s->x = x;
   s->have_x = 1;
   if (first) *first = x;
   return ORC_OK;
+}
+
+/* Prefill whose first generated token is drawn from the full model's
+ * distribution at the given temperature (> 0), with the uniform keyed by the
+ * last prompt position n - 1 (purpose 2, index 0); temperature 0 is
+ * orc_prefill.  *margin receives the draw's margin (orc_draw). */
+int orc_prefill_sampled(orc_sess* s, const int32_t* ids, int n, int trace_T, double temperature,
+                        uint32_t seed, int32_t* first, double* margin) {
+  if (margin) *margin = 0.0;
+  if (!(temperature > 0.0)) return orc_prefill(s, ids, n, trace_T, first);
+  if (n < 1 || trace_T < 1) return ORC_ERR_ARG;
+  if (n + 1 > s->max_seq) return ORC_ERR_CAPACITY;
+  const int V = s->m->c.vocab;
+  s->kv_len = 0;
+  s->have_x = 0;
+  double* z = (double*)malloc(sizeof(double) * 2 * (size_t)V);
+  if (!z) return ORC_ERR_NOMEM;
+  int32_t x = -1;
+  int rc = run_prompt(s, ids, n, trace_T, &x, z);
+  if (rc == ORC_OK) {
+    double mg;
+    orc_tempered(z, V, temperature, z + V);
+    x = orc_draw(z + V, V, uniform_of(seed, n - 1, 2, 0), &mg);
+    if (margin) *margin = mg;
+    s->kv_len = n;
+    s->x = x;
+    s->have_x = 1;
+    if (first) *first = x;
+  }
+  free(z);
+  return rc;
 }
 
 /* Resume from a known sequence: KV for ids[0..n-1), pending token ids[n-1]. */
@@ -645,7 +747,7 @@ int orc_resume(orc_sess* s, const int32_t* ids, int n, int trace_T) {
   if (n > s->max_seq) return ORC_ERR_CAPACITY;
   s->kv_len = 0;
   s->have_x = 0;
-  int rc = run_prompt(s, ids, n - 1, trace_T, NULL);
+  int rc = run_prompt(s, ids, n - 1, trace_T, NULL, NULL);
   if (rc) return rc;
   s->kv_len = n - 1;
   s->x = ids[n - 1];
@@ -667,16 +769,26 @@ int orc_resume(orc_sess* s, const int32_t* ids, int n, int trace_T) {
  *     g_0..g_k (greedy).
  *  4. accept: a = the longest prefix with d_i = g_{i-1}; emit d_1..d_a, g_a.
  *  5. rollback: KV length p + a + 1, pending token g_a, and the full-model
- *     max-probabilities of rows 0..a join the trace. */
+ *     max-probabilities of rows 0..a join the trace.
+ * With temperature T > 0 (speculative sampling, §4.1): d_i is drawn from the
+ * exit distribution at temperature T (uniform U(p, 0, i-1)); step 4 tests
+ * d_1, d_2, ... in turn with orc_spec_step against the full model's row i-1
+ * at temperature T (r = U(p, 1, i-1), u = U(p, 2, 0)) and stops at the first
+ * rejection, whose residual draw is the last emitted token; when all k
+ * drafts are kept, the last token is drawn from row k with U(p, 2, 0).  The
+ * Q-network and the trace still see the exit statistics at temperature 1. */
 int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
   const orc_model* m = s->m;
   const orc_cfg* c = &m->c;
-  int d = c->d_model, L = c->n_layers;
+  int d = c->d_model, L = c->n_layers, V = c->vocab;
   memset(lg, 0, sizeof(*lg));
   if (!s->have_x) return ORC_ERR_STATE;
   if (cap < 1) return ORC_ERR_ARG;
   int rc = check_policy(m, P);
   if (rc) return rc;
+  if (!(P->temperature >= 0.0)) return ORC_ERR_ARG;
+  const int sampled = P->temperature > 0.0;
+  const double Tmp = P->temperature;
   int topk = P->topk > 0 ? P->topk : 5;
   int p = s->kv_len, x = s->x;
   int kcap = 0;
@@ -690,11 +802,27 @@ int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
   lg->pos = p;
   lg->x = x;
   lg->kcap = kcap;
+  lg->sampled = sampled;
 
   int32_t drafts[ORC_MAX_K];
   int k = 0;
   double* h = (double*)malloc(sizeof(double) * (size_t)(kcap + 1) * d);
-  if (!h) return ORC_ERR_NOMEM;
+  /* sampled decoding: exit logits, draft distributions q_1..q_kcap, the
+   * verify rows' distributions and a residual row */
+  double* z = NULL;
+  double* q = NULL;
+  double* pv = NULL;
+  double* res = NULL;
+  if (sampled) {
+    z = (double*)malloc(sizeof(double) * (size_t)V);
+    q = (double*)malloc(sizeof(double) * (size_t)(kcap > 0 ? kcap : 1) * V);
+    pv = (double*)malloc(sizeof(double) * (size_t)(kcap + 1) * V);
+    res = (double*)malloc(sizeof(double) * (size_t)V);
+  }
+  if (!h || (sampled && (!z || !q || !pv || !res))) {
+    rc = ORC_ERR_NOMEM;
+    goto out;
+  }
   if (kcap > 0) {
     int n_c = P->kind == ORC_POLICY_LEDE ? P->n_cand : 1;
     int done = 0, lstar = 0, keep = 0;
@@ -704,7 +832,7 @@ int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
       rc = orc_forward(s, &x, 1, p, done, cj, h);
       if (rc) goto out;
       done = cj;
-      rc = orc_exit_head(m, h, NULL, topk, &st);
+      rc = orc_exit_head(m, h, z, topk, &st);
       if (rc) goto out;
       lg->visited[lg->n_visited++] = cj;
       int act, aq = 1;
@@ -723,16 +851,27 @@ int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
       }
     }
     lg->lstar = lstar;
-    drafts[0] = st.argmax;
-    lg->draft_margin[0] = st.margin;
+    if (sampled) {
+      orc_tempered(z, V, Tmp, q);
+      drafts[0] = orc_draw(q, V, uniform_of(P->sample_seed, p, 0, 0), &lg->draft_margin[0]);
+    } else {
+      drafts[0] = st.argmax;
+      lg->draft_margin[0] = st.margin;
+    }
     k = 1;
     while (k < kcap && keep) {
       rc = orc_forward(s, &drafts[k - 1], 1, p + k, 0, lstar, h);
       if (rc) goto out;
-      rc = orc_exit_head(m, h, NULL, topk, &st);
+      rc = orc_exit_head(m, h, z, topk, &st);
       if (rc) goto out;
-      drafts[k] = st.argmax;
-      lg->draft_margin[k] = st.margin;
+      if (sampled) {
+        orc_tempered(z, V, Tmp, q + (int64_t)k * V);
+        drafts[k] = orc_draw(q + (int64_t)k * V, V, uniform_of(P->sample_seed, p, 0, k),
+                             &lg->draft_margin[k]);
+      } else {
+        drafts[k] = st.argmax;
+        lg->draft_margin[k] = st.margin;
+      }
       ++k;
       if (P->kind == ORC_POLICY_THRESHOLD)
         keep = threshold_decide(P, &st, lg);
@@ -753,24 +892,49 @@ int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
     if (rc) goto out;
     for (int i = 0; i <= k; ++i) {
       orc_stats st;
-      rc = orc_exit_head(m, h + (int64_t)i * d, NULL, 1, &st);
+      rc = orc_exit_head(m, h + (int64_t)i * d, z, 1, &st);
       if (rc) goto out;
       lg->verify_tok[i] = st.argmax;
       lg->verify_margin[i] = st.margin;
       lg->verify_pmax[i] = st.pmax;
+      if (sampled) orc_tempered(z, V, Tmp, pv + (int64_t)i * V);
     }
-    int a = 0;
-    while (a < k && drafts[a] == lg->verify_tok[a]) ++a;
+    int a = 0, last;
+    if (sampled) {
+      last = -1;
+      while (a < k) {
+        int kept;
+        const int t = orc_spec_step(pv + (int64_t)a * V, q + (int64_t)a * V, V, drafts[a],
+                                    uniform_of(P->sample_seed, p, 1, a),
+                                    uniform_of(P->sample_seed, p, 2, 0), res, &kept,
+                                    &lg->accept_margin[a], &lg->fix_margin);
+        if (!kept) {
+          last = t;
+          break;
+        }
+        ++a;
+      }
+      if (last < 0)
+        last = orc_draw(pv + (int64_t)k * V, V, uniform_of(P->sample_seed, p, 2, 0),
+                        &lg->fix_margin);
+    } else {
+      while (a < k && drafts[a] == lg->verify_tok[a]) ++a;
+      last = lg->verify_tok[a];
+    }
     lg->a = a;
     for (int i = 0; i < a; ++i) lg->emitted[i] = drafts[i];
-    lg->emitted[a] = lg->verify_tok[a];
+    lg->emitted[a] = last;
     lg->n_emit = a + 1;
     s->kv_len = p + a + 1;
-    s->x = lg->verify_tok[a];
+    s->x = last;
     for (int i = 0; i <= a; ++i) orc_trace_push(s, lg->verify_pmax[i]);
   }
 out:
   free(h);
+  free(z);
+  free(q);
+  free(pv);
+  free(res);
   return rc;
 }
 

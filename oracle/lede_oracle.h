@@ -61,6 +61,8 @@ typedef struct {
   const float* q_params;             /* W1[h][in], b1[h], W2[2][h], b2[2] */
   int32_t fixed_k;                   /* LEDE: 0 adaptive drafting; > 0 fixed draft length */
   double conf_threshold;             /* THRESHOLD: drafting goes on while pmax >= this */
+  double temperature;                /* 0: greedy; > 0: speculative sampling at this temperature */
+  uint32_t sample_seed;              /* key of the uniforms (synth_sample_uniform) */
 } orc_policy;
 
 typedef struct {
@@ -75,6 +77,9 @@ typedef struct {
   double verify_pmax[ORC_MAX_K + 1];
   double q_val[ORC_MAX_Q][2];
   double q_state[ORC_MAX_Q][3];
+  int32_t sampled;                   /* 1 when the round sampled (temperature > 0) */
+  double accept_margin[ORC_MAX_K];   /* (p(d) - r q(d)) / max(p(d), r q(d)); > 0 accepts */
+  double fix_margin;                 /* distance of the last draw to a CDF boundary / mass */
 } orc_round_log;
 
 typedef struct orc_model orc_model;
@@ -102,6 +107,12 @@ void orc_qnet(const float* params, int in, int hidden, const double* s, double q
 double orc_trace_conf(const orc_sess* s, int T);
 void orc_trace_push(orc_sess* s, double pmax);
 int orc_prefill(orc_sess* s, const int32_t* ids, int n, int trace_T, int32_t* first);
+int orc_prefill_sampled(orc_sess* s, const int32_t* ids, int n, int trace_T, double temperature,
+                        uint32_t seed, int32_t* first, double* margin);
+void orc_tempered(const double* z, int V, double temperature, double* p);
+int orc_draw(const double* w, int V, double u, double* margin);
+int orc_spec_step(const double* p, const double* q, int V, int d, double r, double u,
+                  double* res, int* accepted, double* accept_margin, double* draw_margin);
 int orc_resume(orc_sess* s, const int32_t* ids, int n, int trace_T);
 int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg);
 int orc_generate(orc_sess* s, const orc_policy* P, int n_new, int32_t* out, orc_round_log* logs,

@@ -36,6 +36,8 @@ struct DevPolicy {
   int32_t cand[kMaxCand];
   int32_t fixed_k;  // LEDE: fixed draft length (0: adaptive)
   float tau;        // THRESHOLD: confidence threshold on a draft's max-probability
+  float temp;       // sampled decoding temperature (0: greedy)
+  uint32_t seed;    // sampled decoding seed
 };
 
 // Per-row statistics of an exit distribution (mirrors ssd_exit_stats).
@@ -59,6 +61,7 @@ struct Ctl {
   int32_t trace_n, trace_head;
   float trace[kTraceCap];  // ring of full-model max-probabilities
   DevPolicy pol;
+  float dq_zmax[kMaxDraft], dq_sum[kMaxDraft];  // sampled drafts: max logit, normaliser
   ssd_round_trace cur;     // record of the round in flight
 };
 
@@ -165,6 +168,7 @@ struct Bufs {
   float* attn_ml;    // [kMaxM][Hq][nsplit][2] partial (max, sum)
   uint32_t* attn_counter;  // [Hkv][kMaxM] split tickets of the attention merge
   uint32_t* chain_bar;     // [2] grid-wide phase arrivals / blocks done of the chain kernel
+  float* draft_logits;     // [kMaxDraft][V] exit logits of each draft (sampled decoding)
   float* attn_out;   // [kMaxM][qd]
   float* act;        // [kMaxM][F]
   float* logits;     // [kMaxM][V] (written only when requested)

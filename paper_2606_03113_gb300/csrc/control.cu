@@ -31,6 +31,141 @@ __device__ float trace_conf(const Ctl* c, int T) {
   return -acc / (float)n;
 }
 
+// ------------------------------------------------- sampled decoding (§4.1)
+// Speculative sampling draws drafts from the exit distribution and emitted
+// tokens from the full model's, both at temperature T:
+// P(v) = exp((z_v - max z) / T) / sum_w exp((z_w - max z) / T).
+// Every reduction below runs in a fixed order (contiguous per-thread chunks
+// of the vocabulary, chunk sums added in chunk order by one thread), so a
+// draw depends only on the logits and the uniform, never on scheduling.
+// The uniforms come from synth_sample_uniform keyed by the round's pending
+// position: purpose 0 the draw of draft i, 1 the acceptance test of draft i,
+// 2 the round's last draw.
+
+constexpr int kSampleThreads = 256;  // block size of k_decide and k_accept
+
+struct SampleSmem {
+  float part[kSampleThreads];  // chunk sums, then their exclusive prefix
+  float red[kSampleThreads / 32];
+  float total, zmax;
+  int tok;
+  float margin;
+};
+
+__device__ __forceinline__ void chunk_of(int V, int& v0, int& v1) {
+  const int C = (V + (int)blockDim.x - 1) / (int)blockDim.x;
+  v0 = min(V, (int)threadIdx.x * C);
+  v1 = min(V, v0 + C);
+}
+
+// Maximum of z[0..V) broadcast to the block (exact in any order).
+__device__ float block_zmax(const float* __restrict__ z, int V, SampleSmem& sm) {
+  int v0, v1;
+  chunk_of(V, v0, v1);
+  float m = -INFINITY;
+  for (int v = v0; v < v1; ++v) m = fmaxf(m, z[v]);
+  m = warp_max(m);
+  if ((threadIdx.x & 31) == 0) sm.red[threadIdx.x >> 5] = m;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float r = sm.red[0];
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) r = fmaxf(r, sm.red[w]);
+    sm.zmax = r;
+  }
+  __syncthreads();
+  const float r = sm.zmax;
+  __syncthreads();
+  return r;
+}
+
+// Sum of w(v) over [0, V) in the fixed chunk order; leaves the exclusive
+// prefix of the chunk sums in sm.part and returns the total to every thread.
+template <typename W>
+__device__ float block_chunk_sums(int V, W w, SampleSmem& sm) {
+  int v0, v1;
+  chunk_of(V, v0, v1);
+  float acc = 0.f;
+  for (int v = v0; v < v1; ++v) acc += w(v);
+  sm.part[threadIdx.x] = acc;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float c = 0.f;
+    for (int i = 0; i < (int)blockDim.x; ++i) {
+      const float x = sm.part[i];
+      sm.part[i] = c;
+      c += x;
+    }
+    sm.total = c;
+  }
+  __syncthreads();
+  return sm.total;
+}
+
+// Inverse-CDF draw from non-negative weights w(v): with W the total and
+// C_v = w(0) + ... + w(v) in token order, the token is the first v with
+// C_v > u W; *margin = min(u W - C_{v-1}, C_v - u W) / W.  Returns -1 when W
+// is not positive; when rounding leaves u W at or beyond the total, the last
+// token of positive weight (margin 0).  Every thread of the block calls it.
+template <typename W>
+__device__ int block_draw(int V, W w, float u, float* margin, SampleSmem& sm) {
+  const float S = block_chunk_sums(V, w, sm);
+  int v0, v1;
+  chunk_of(V, v0, v1);
+  if (threadIdx.x == 0) {
+    sm.tok = -1;
+    sm.margin = 0.f;
+  }
+  __syncthreads();
+  if (S > 0.f) {
+    const float T = u * S;
+    const float lo = sm.part[threadIdx.x];
+    const float hi = threadIdx.x + 1 < blockDim.x ? sm.part[threadIdx.x + 1] : S;
+    // chunk intervals [lo, hi) are disjoint: at most one thread holds T
+    if (v1 > v0 && T >= lo && T < hi) {
+      float c = lo, mg = 0.f;
+      int found = -1, last = -1;
+      for (int v = v0; v < v1; ++v) {
+        const float wv = w(v);
+        const float nx = c + wv;
+        if (wv > 0.f) last = v;
+        if (nx > T) {
+          found = v;
+          mg = fminf(T - c, nx - T) / S;
+          break;
+        }
+        c = nx;
+      }
+      sm.tok = found >= 0 ? found : last;
+      sm.margin = found >= 0 ? mg : 0.f;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && S > 0.f && sm.tok < 0) {
+    int v = V - 1;
+    while (v > 0 && !(w(v) > 0.f)) --v;
+    sm.tok = v;
+    sm.margin = 0.f;
+  }
+  __syncthreads();
+  const int tok = sm.tok;
+  if (margin) *margin = sm.margin;
+  __syncthreads();
+  return tok;
+}
+
+struct Tempered {
+  const float* z;
+  float zmax, temp;
+  __device__ float operator()(int v) const { return expf((z[v] - zmax) / temp); }
+};
+
+// Weights of the residual max(0, p - q) of one acceptance test.
+struct Residual {
+  Tempered p, q;
+  float sp, sq;  // normalisers of p and q
+  __device__ float operator()(int v) const { return fmaxf(p(v) / sp - q(v) / sq, 0.f); }
+};
+
 // h[m] = embed[token_m] (fp32) and the row's sum of squares for the first
 // RMSNorm.  One block per row.  Optionally sets the drafting switch handle to
 // the chosen exit-layer index.
@@ -122,6 +257,9 @@ __global__ void k_round_begin(Dims D, Bufs B, cudaGraphConditionalHandle draft_i
   r.a = 0;
   r.n_emit = 0;
   r.n_q = 0;
+  r.sampled = P.temp > 0.f ? 1 : 0;
+  for (int i = 0; i < SSD_TRACE_MAXK; ++i) r.accept_margin[i] = 0.f;
+  r.fix_margin = 0.f;
   set_cond(draft_if, kcap > 0 ? 1u : 0u);
 }
 
@@ -189,6 +327,45 @@ __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, in
       q1 += b2[1];
     }
   }
+  // Draft token of this decision: argmax of the exit distribution (greedy)
+  // or a draw from it at the policy's temperature (sampled decoding).
+  __shared__ int s_slot, s_tok;
+  __shared__ float s_margin;
+  __shared__ SampleSmem sm;
+  const bool sampled = P.temp > 0.f;
+  if (tid == 0) {
+    const int aq = use_q ? (q1 > q0 ? 1 : 0) : 1;
+    int slot = -1;
+    if (mode == kDecideWalk) {
+      if (is_last || aq) slot = 0;
+    } else {
+      const int k = c->k;
+      if (k >= 1 && k < c->kcap && k < kMaxDraft) slot = k;
+    }
+    s_slot = slot;
+    s_tok = st.argmax;
+    s_margin = st.margin;
+  }
+  if (sampled) {
+    __syncthreads();
+    const int slot = s_slot;
+    if (slot >= 0) {
+      const float* z = B.logits;  // row 0: this exit's logits
+      float* keep = B.draft_logits + (size_t)slot * D.V;
+      for (int v = tid; v < D.V; v += blockDim.x) keep[v] = z[v];
+      const float zmax = block_zmax(z, D.V, sm);
+      const Tempered q{z, zmax, P.temp};
+      float mg = 0.f;
+      const int d = block_draw(D.V, q, synth_sample_uniform(P.seed, (uint32_t)c->pos, 0u,
+                                                            (uint32_t)slot), &mg, sm);
+      if (tid == 0) {
+        c->dq_zmax[slot] = zmax;
+        c->dq_sum[slot] = sm.total;
+        s_tok = d;
+        s_margin = mg;
+      }
+    }
+  }
   if (tid != 0) return;
   ssd_round_trace& r = c->cur;
   const int aq = use_q ? (q1 > q0 ? 1 : 0) : 1;
@@ -203,7 +380,10 @@ __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, in
     r.q_state[i][1] = use_q ? s_state[1] : st.entropy;
     r.q_state[i][2] = use_q ? s_state[2] : 0.f;
   }
-  if (st.argmax < 0 || st.argmax >= D.V) atomicOr(&c->err, (int)kErrToken);
+  const int dtok = s_tok;
+  if (st.argmax < 0 || st.argmax >= D.V || dtok < 0 || dtok >= D.V) {
+    atomicOr(&c->err, (int)kErrToken);
+  }
   if (mode == kDecideWalk) {
     if (r.n_visited < SSD_TRACE_MAXC) r.visited[r.n_visited++] = layer;
     const int act = is_last ? 1 : aq;
@@ -211,9 +391,9 @@ __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, in
       c->lstar = layer;
       c->lstar_idx = cand_idx;
       c->k = 1;
-      c->tok[1] = st.argmax;
-      r.drafts[0] = st.argmax;
-      r.draft_margin[0] = st.margin;
+      c->tok[1] = dtok;
+      r.drafts[0] = dtok;
+      r.draft_margin[0] = s_margin;
       c->keep = (go && 1 < c->kcap) ? 1 : 0;
       set_cond(next_if, 0u);
     } else {
@@ -227,9 +407,9 @@ __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, in
       set_cond(draft_while, 0u);
       return;
     }
-    c->tok[k + 1] = st.argmax;
-    r.drafts[k] = st.argmax;
-    r.draft_margin[k] = st.margin;
+    c->tok[k + 1] = dtok;
+    r.drafts[k] = dtok;
+    r.draft_margin[k] = s_margin;
     c->k = k + 1;
     c->keep = (go && k + 1 < c->kcap) ? 1 : 0;
     set_cond(draft_while, (unsigned)c->keep);
@@ -242,31 +422,95 @@ __global__ void k_draft_begin(Bufs B, cudaGraphConditionalHandle draft_while) {
   set_cond(draft_while, (unsigned)B.ctl->keep);
 }
 
-// Greedy verification (§4.1: greedy decoding, speculative acceptance):
-// g_i = argmax of verify row i; a = longest prefix with d_i = g_{i-1}; emit
-// d_1..d_a and g_a; KV length becomes pos + a + 1 (rows beyond it are stale
-// and rewritten before any read); the full model's max-probabilities of rows
-// 0..a join the C_trace window; g_a is the next pending token.
+// Verification and acceptance (§4.1: speculative acceptance), one round.
+// Greedy (temperature 0): g_i = argmax of verify row i; a = the longest
+// prefix with d_i = g_{i-1}; emit d_1..d_a and g_a.
+// Sampled (temperature T > 0): p_i = the full model's row i at T, q_i = the
+// exit distribution d_i was drawn from; d_1, d_2, ... are tested in turn and
+// d_i is kept when r_i q_i(d_i) < p_{i-1}(d_i) (probability min(1, p/q));
+// the first rejected test ends the round with a draw from the residual
+// max(0, p_{i-1} - q_i) (from p_{i-1} should it carry no mass); when all k
+// are kept, the last token is drawn from p_k.  The emitted tokens then
+// follow the full model's distribution at T whatever the drafts were.
+// Either way the KV length becomes pos + a + 1 (rows beyond it are stale and
+// rewritten before any read), the full model's max-probabilities of rows
+// 0..a join the C_trace window and the last emitted token is the next
+// pending token.
 __global__ void k_accept(Dims D, Bufs B, cudaGraphConditionalHandle gen_while) {
   pdl_wait();
   pdl_launch_dependents();
+  __shared__ SampleSmem sm;
+  __shared__ int s_a, s_last;
   Ctl* c = B.ctl;
   ssd_round_trace& r = c->cur;
+  const DevPolicy& P = c->pol;
+  const bool sampled = P.temp > 0.f;
   const int k = c->k;
-  int a = 0;
-  while (a < k && c->tok[a + 1] == B.stats[a].argmax) ++a;
+  if (sampled) {
+    const uint32_t pos = (uint32_t)c->pos;
+    const float u_last = synth_sample_uniform(P.seed, pos, 2u, 0u);
+    int a = 0, last = -1;
+    float fix = 0.f;
+    while (a < k && a < kMaxDraft) {
+      const float* zp = B.logits + (size_t)a * D.V;
+      const float* zq = B.draft_logits + (size_t)a * D.V;
+      const float zmp = block_zmax(zp, D.V, sm);
+      const Tempered pt{zp, zmp, P.temp};
+      const float sp = block_chunk_sums(D.V, pt, sm);
+      const Tempered qt{zq, c->dq_zmax[a], P.temp};
+      const float sq = c->dq_sum[a];
+      const int d = c->tok[a + 1];
+      const bool ok_d = d >= 0 && d < D.V && sp > 0.f && sq > 0.f;
+      const float pd = ok_d ? pt(d) / sp : 0.f;
+      const float qd = ok_d ? qt(d) / sq : 0.f;
+      const float rq = synth_sample_uniform(P.seed, pos, 1u, (uint32_t)a) * qd;
+      const float den = fmaxf(pd, rq);
+      if (threadIdx.x == 0) r.accept_margin[a] = den > 0.f ? (pd - rq) / den : 0.f;
+      if (ok_d && rq < pd) {
+        ++a;
+        continue;
+      }
+      const Residual res{pt, qt, sp, sq};
+      last = block_draw(D.V, res, u_last, &fix, sm);
+      if (last < 0) last = block_draw(D.V, pt, u_last, &fix, sm);
+      break;
+    }
+    if (last < 0) {
+      const float* zp = B.logits + (size_t)a * D.V;
+      const float zmp = block_zmax(zp, D.V, sm);
+      last = block_draw(D.V, Tempered{zp, zmp, P.temp}, u_last, &fix, sm);
+    }
+    if (threadIdx.x == 0) {
+      s_a = a;
+      s_last = last;
+      r.fix_margin = fix;
+    }
+  }
+  if (threadIdx.x != 0) return;
+  int a = 0, g;
+  if (sampled) {
+    a = s_a;
+    g = s_last;
+    if (g < 0 || g >= D.V) {
+      atomicOr(&c->err, (int)kErrToken);
+      g = 0;
+    }
+  } else {
+    while (a < k && c->tok[a + 1] == B.stats[a].argmax) ++a;
+    g = B.stats[a].argmax;
+  }
   for (int i = 0; i <= k; ++i) {
     r.verify_tok[i] = B.stats[i].argmax;
     r.verify_margin[i] = B.stats[i].margin;
     r.verify_pmax[i] = B.stats[i].pmax;
   }
-  const int g = B.stats[a].argmax;
   for (int i = 0; i < a; ++i) r.emitted[i] = c->tok[i + 1];
   r.emitted[a] = g;
   for (int i = 0; i <= a; ++i) {
     if (c->n_out + i < D.max_seq) B.out_tok[c->n_out + i] = r.emitted[i];
     trace_push(c, B.stats[i].pmax);
   }
+  r.sampled = sampled ? 1 : 0;
   r.lstar = c->lstar;
   r.k = k;
   r.a = a;
@@ -309,12 +553,29 @@ __global__ void k_trace_push(Bufs B, int first_row, int n_rows) {
   for (int i = 0; i < n_rows; ++i) trace_push(B.ctl, B.stats[first_row + i].pmax);
 }
 
-// Pending token = argmax of stats[row] (token < 0) or the given token.
-__global__ void k_set_pending(Bufs B, int row, int token, int pos) {
+// Pending token after a prompt: the given token, or (token < 0) the argmax
+// of stats[row], or with a sampling temperature a draw from logits row `row`
+// keyed by the last prompt position pos - 1 (purpose 2, index 0).
+__global__ void k_set_pending(Dims D, Bufs B, int row, int token, int pos) {
   pdl_wait();
   pdl_launch_dependents();
+  __shared__ SampleSmem sm;
   Ctl* c = B.ctl;
-  c->x = token >= 0 ? token : B.stats[row].argmax;
+  const DevPolicy& P = c->pol;
+  int x = token;
+  if (token < 0 && P.temp > 0.f) {
+    const float* z = B.logits + (size_t)row * D.V;
+    const float zmax = block_zmax(z, D.V, sm);
+    x = block_draw(D.V, Tempered{z, zmax, P.temp},
+                   synth_sample_uniform(P.seed, (uint32_t)(pos - 1), 2u, 0u), nullptr, sm);
+  }
+  if (threadIdx.x != 0) return;
+  if (token < 0 && !(P.temp > 0.f)) x = B.stats[row].argmax;
+  if (x < 0 || x >= D.V) {
+    atomicOr(&c->err, (int)kErrToken);
+    x = 0;
+  }
+  c->x = x;
   c->pos = pos;
 }
 
@@ -387,8 +648,8 @@ cudaError_t launch_round_begin(const Dims& D, const Bufs& B, cudaGraphConditiona
 cudaError_t launch_decide(const Dims& D, const Bufs& B, int mode, int cand_idx, int is_last,
                           int layer, cudaGraphConditionalHandle next_if,
                           cudaGraphConditionalHandle draft_while, cudaStream_t st) {
-  return launch_ex(k_decide, dim3(1), dim3(256), 0, st, D, B, mode, cand_idx, is_last, layer,
-                   next_if, draft_while);
+  return launch_ex(k_decide, dim3(1), dim3(kSampleThreads), 0, st, D, B, mode, cand_idx, is_last,
+                   layer, next_if, draft_while);
 }
 
 cudaError_t launch_draft_begin(const Bufs& B, cudaGraphConditionalHandle draft_while,
@@ -398,7 +659,7 @@ cudaError_t launch_draft_begin(const Bufs& B, cudaGraphConditionalHandle draft_w
 
 cudaError_t launch_accept(const Dims& D, const Bufs& B, cudaGraphConditionalHandle gen_while,
                           cudaStream_t st) {
-  return launch_ex(k_accept, dim3(1), dim3(1), 0, st, D, B, gen_while);
+  return launch_ex(k_accept, dim3(1), dim3(kSampleThreads), 0, st, D, B, gen_while);
 }
 
 cudaError_t launch_begin_call(const Bufs& B, int max_new, cudaStream_t st) {
@@ -413,8 +674,10 @@ cudaError_t launch_trace_push(const Bufs& B, int first_row, int n_rows, cudaStre
   return launch_ex(k_trace_push, dim3(1), dim3(1), 0, st, B, first_row, n_rows);
 }
 
-cudaError_t launch_set_pending(const Bufs& B, int stats_row, int token, int pos, cudaStream_t st) {
-  return launch_ex(k_set_pending, dim3(1), dim3(1), 0, st, B, stats_row, token, pos);
+cudaError_t launch_set_pending(const Dims& D, const Bufs& B, int stats_row, int token, int pos,
+                               cudaStream_t st) {
+  return launch_ex(k_set_pending, dim3(1), dim3(kSampleThreads), 0, st, D, B, stats_row, token,
+                   pos);
 }
 
 cudaError_t launch_qnet_eval(const Bufs& B, int hidden, const float* states, int n, float* q,

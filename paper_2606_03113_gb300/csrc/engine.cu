@@ -2,7 +2,8 @@
 // validation, prefill, and the CUDA graphs that run speculation rounds with
 // every decision taken on the device.
 //
-// Round graph (one speculation round, §3.3; greedy acceptance, §4.1):
+// Round graph (one speculation round, §3.3; greedy or speculative-sampling
+// acceptance, §4.1):
 //   round_begin ─ IF(kcap > 0) { walk ; draft_begin ; WHILE(keep) { draft } } ─ verify ─ accept
 //   walk  = embed(x) · layers(1..c_1) · head · decide_1 ·
 //           IF(continue) { layers(c_1+1..c_2) · head · decide_2 · IF(continue) { ... } }
@@ -85,6 +86,7 @@ size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
   b.attn_out = cv.take<float>(sizeof(float) * kMaxM * d.qd);
   b.act = cv.take<float>(sizeof(float) * kMaxM * d.F);
   b.logits = cv.take<float>(sizeof(float) * kMaxM * (size_t)d.V);
+  b.draft_logits = cv.take<float>(sizeof(float) * kMaxDraft * (size_t)d.V);
   b.head_part = cv.take<void>(sizeof(HeadPart) * kMaxM * 2 * (size_t)kMaxBlocks);
   b.head_counter = cv.take<uint32_t>(sizeof(uint32_t));
   b.stats = cv.take<RowStats>(sizeof(RowStats) * kMaxM);
@@ -138,6 +140,7 @@ struct ssd_ctx {
   int kind = SSD_POLICY_AR;
   std::vector<int> cand;
   int kmax = 0, static_l = 0, static_k = 0, q_hidden = 0, trace_T = 20, topk = 5, fixed_k = 0;
+  bool sampled = false;  // temperature > 0: the exit heads write their logits
   // graphs
   cudaGraph_t round_g = nullptr, gen_g = nullptr;
   cudaGraphExec_t round_x = nullptr, gen_x = nullptr;
@@ -263,7 +266,7 @@ cudaError_t build_walk(ssd_ctx* x, Seq& s, const std::vector<int>& cands, int j,
   GK(s.begin());
   if (j == 0) GK(launch_embed(x->D, x->B, x->cfg.dtype, x->embed, rows(kRowsWalk), false, 0, x->cap));
   GK(enqueue_layers(x, done, cands[j], rows(kRowsWalk), 1, x->cap));
-  GK(enqueue_head(x, rows(kRowsWalk), 1, x->topk, false, x->cap));
+  GK(enqueue_head(x, rows(kRowsWalk), 1, x->topk, x->sampled, x->cap));
   GK(launch_decide(x->D, x->B, kDecideWalk, j, last ? 1 : 0, cands[j], next, 0, x->cap));
   GK(s.end());
   if (last) return cudaSuccess;
@@ -307,7 +310,7 @@ cudaError_t build_draft_phase(ssd_ctx* x, cudaGraph_t body) {
     GK(launch_embed(x->D, x->B, x->cfg.dtype, x->embed, rows(kRowsDraft), false, 0, x->cap));
     GK(enqueue_layers(x, 0, cands[0], rows(kRowsDraft), 1, x->cap));
   }
-  GK(enqueue_head(x, rows(kRowsDraft), 1, x->topk, false, x->cap));
+  GK(enqueue_head(x, rows(kRowsDraft), 1, x->topk, x->sampled, x->cap));
   GK(launch_decide(x->D, x->B, kDecideDraft, 0, 0, 0, 0, hw, x->cap));
   return w.end();
 }
@@ -331,7 +334,7 @@ cudaError_t build_round(ssd_ctx* x, cudaGraph_t g, cudaGraphConditionalHandle ge
   GK(launch_embed(x->D, x->B, x->cfg.dtype, x->embed, rows(kRowsVerify), spec, 0, x->cap));
   const int mrows = spec ? std::min(x->kmax + 1, kMaxM) : 1;
   GK(enqueue_layers(x, 0, x->D.L, rows(kRowsVerify), mrows, x->cap));
-  GK(enqueue_head(x, rows(kRowsVerify), mrows, x->topk, false, x->cap));
+  GK(enqueue_head(x, rows(kRowsVerify), mrows, x->topk, x->sampled, x->cap));
   GK(launch_accept(x->D, x->B, gen, x->cap));
   return s.end();
 }
@@ -388,7 +391,7 @@ ssd_status run_prompt(ssd_ctx* x, int n) {
     CK(x, launch_embed(x->D, x->B, x->cfg.dtype, x->embed, sel, true, 0, x->stream));
     CK(x, enqueue_layers(x, 0, x->D.L, sel, kPrefillChunk, x->stream));
     if (c0 + M > n - T || c0 + M == n) {
-      CK(x, enqueue_head(x, sel, kPrefillChunk, x->topk, false, x->stream));
+      CK(x, enqueue_head(x, sel, kPrefillChunk, x->topk, x->sampled, x->stream));
       const int first = std::max(c0, n - T) - c0;
       if (first < M) CK(x, launch_trace_push(x->B, first, M - first, x->stream));
     }
@@ -552,6 +555,8 @@ ssd_status ssd_set_policy(ssd_ctx* x, const ssd_policy* p) {
     if (p->static_l < 1 || p->static_l > L || p->static_k < 1)
       return fail(x, SSD_ERR_INVALID_ARG, "static_l must be in 1..n_layers and static_k >= 1");
   }
+  if (!(p->temperature >= 0.f && p->temperature <= 100.f))
+    return fail(x, SSD_ERR_INVALID_ARG, "temperature must be in [0, 100]");
   if (p->kind == SSD_POLICY_THRESHOLD) {
     if (p->static_l < 1 || p->static_l > L)
       return fail(x, SSD_ERR_INVALID_ARG, "static_l must be in 1..n_layers");
@@ -581,20 +586,32 @@ ssd_status ssd_set_policy(ssd_ctx* x, const ssd_policy* p) {
   dp.q_hidden = p->kind == SSD_POLICY_LEDE ? p->qnet_hidden : 0;
   dp.fixed_k = p->kind == SSD_POLICY_LEDE ? p->fixed_k : 0;
   dp.tau = p->kind == SSD_POLICY_THRESHOLD ? p->conf_threshold : 0.f;
+  dp.temp = p->temperature;
+  dp.seed = p->sample_seed;
   CK(x, cudaMemcpyAsync(&x->B.ctl->pol, &dp, sizeof(dp), cudaMemcpyHostToDevice, x->stream));
   if (p->kind == SSD_POLICY_LEDE)
     CK(x, cudaMemcpyAsync(x->B.qparams, p->qnet_params, sizeof(float) * (6 * p->qnet_hidden + 2),
                           cudaMemcpyHostToDevice, x->stream));
   CK(x, cudaStreamSynchronize(x->stream));
+  // The graphs depend on the policy kind, the candidate (or static) exit
+  // layers, kmax, topk and whether the heads write logits; everything else
+  // is read on the device from the policy just copied.
+  const int kmax_new = p->kind == SSD_POLICY_AR ? 0 : p->kmax;
+  const bool sampled = p->temperature > 0.f;
+  const bool same_graphs = x->have_policy && x->kind == p->kind && x->cand == cand &&
+                           x->kmax == kmax_new && x->static_l == p->static_l &&
+                           x->topk == dp.topk && x->sampled == sampled;
   x->kind = p->kind;
   x->cand = cand;
-  x->kmax = p->kind == SSD_POLICY_AR ? 0 : p->kmax;
+  x->kmax = kmax_new;
   x->static_l = p->static_l;
   x->static_k = p->static_k;
   x->fixed_k = dp.fixed_k;
   x->q_hidden = dp.q_hidden;
   x->trace_T = dp.trace_T;
   x->topk = dp.topk;
+  x->sampled = sampled;
+  if (same_graphs) return SSD_OK;
   cudaError_t e = build_graphs(x);
   if (e != cudaSuccess) {
     destroy_graphs(x);
@@ -616,7 +633,7 @@ ssd_status ssd_prefill(ssd_ctx* x, const int32_t* ids, int32_t n, int32_t* first
   ssd_status s = run_prompt(x, n);
   if (s) return s;
   const int last_M = (n - 1) % kPrefillChunk + 1;
-  CK(x, launch_set_pending(x->B, last_M - 1, -1, n, x->stream));
+  CK(x, launch_set_pending(x->D, x->B, last_M - 1, -1, n, x->stream));
   Ctl c;
   if ((s = read_ctl(x, &c))) return s;
   CK(x, cudaStreamSynchronize(x->stream));
@@ -638,7 +655,7 @@ ssd_status ssd_resume(ssd_ctx* x, const int32_t* ids, int32_t n) {
                         x->stream));
   ssd_status s = run_prompt(x, n - 1);
   if (s) return s;
-  CK(x, launch_set_pending(x->B, 0, ids[n - 1], n - 1, x->stream));
+  CK(x, launch_set_pending(x->D, x->B, 0, ids[n - 1], n - 1, x->stream));
   Ctl c;
   if ((s = read_ctl(x, &c))) return s;
   CK(x, cudaStreamSynchronize(x->stream));

@@ -73,7 +73,8 @@ cudaError_t launch_accept(const Dims& D, const Bufs& B, cudaGraphConditionalHand
 cudaError_t launch_begin_call(const Bufs& B, int max_new, cudaStream_t st);
 cudaError_t launch_reset_sequence(const Bufs& B, cudaStream_t st);
 cudaError_t launch_trace_push(const Bufs& B, int first_row, int n_rows, cudaStream_t st);
-cudaError_t launch_set_pending(const Bufs& B, int stats_row, int token, int pos, cudaStream_t st);
+cudaError_t launch_set_pending(const Dims& D, const Bufs& B, int stats_row, int token, int pos,
+                               cudaStream_t st);
 cudaError_t launch_qnet_eval(const Bufs& B, int hidden, const float* states, int n, float* q,
                              cudaStream_t st);
 cudaError_t launch_gemv_plain(const Dims& D, const Bufs& B, int dtype, const void* W, int rows,

@@ -101,36 +101,43 @@ class Engine:
     # ----------------------------------------------------------- policies
     def set_policy(self, kind: int, cand=(), kmax: int = 0, static_l: int = 0, static_k: int = 0,
                    qnet_params: np.ndarray | None = None, qnet_hidden: int = 0, trace_T: int = 20,
-                   topk: int = 5, fixed_k: int = 0, conf_threshold: float = 0.0):
+                   topk: int = 5, fixed_k: int = 0, conf_threshold: float = 0.0,
+                   temperature: float = 0.0, sample_seed: int = 0):
+        """temperature > 0 turns on speculative sampling at that temperature
+        (drafts drawn from the exit distribution, emitted tokens distributed
+        as the full model's), with uniforms keyed by sample_seed."""
         cand_arr = (C.c_int32 * max(1, len(cand)))(*cand)
         qp = None
         if qnet_params is not None:
             self._qp = np.ascontiguousarray(qnet_params, dtype=np.float32)
             qp = self._qp.ctypes.data_as(C.POINTER(C.c_float))
         p = S.ssd_policy(kind, len(cand), C.cast(cand_arr, C.POINTER(C.c_int32)), kmax, static_l,
-                         static_k, 3, qnet_hidden, qp, trace_T, topk, fixed_k, conf_threshold)
+                         static_k, 3, qnet_hidden, qp, trace_T, topk, fixed_k, conf_threshold,
+                         temperature, sample_seed)
         S.ssd_set_policy(self.ctx, p)
         self.policy_kind = kind
         self.kmax = 0 if kind == S.SSD_POLICY_AR else kmax
 
-    def set_ar(self):
-        self.set_policy(S.SSD_POLICY_AR)
+    # Each setter takes temperature= and sample_seed= (sampled decoding).
+    def set_ar(self, **sampling):
+        self.set_policy(S.SSD_POLICY_AR, **sampling)
 
-    def set_static(self, l: int, k: int, kmax: int | None = None):
-        self.set_policy(S.SSD_POLICY_STATIC, kmax=kmax or k, static_l=l, static_k=k)
+    def set_static(self, l: int, k: int, kmax: int | None = None, **sampling):
+        self.set_policy(S.SSD_POLICY_STATIC, kmax=kmax or k, static_l=l, static_k=k, **sampling)
 
     def set_lede(self, w: Workload, qnet_params: np.ndarray | None = None, kmax: int | None = None,
-                 cand=None, fixed_k: int = 0):
+                 cand=None, fixed_k: int = 0, **sampling):
         """LEDE (§3.3); one candidate is the ablation without dynamic exit,
         fixed_k > 0 the one without adaptive drafting (Table 3)."""
         qp = qnet_params if qnet_params is not None else synth.qnet_hidden_params(3, w.qnet_hidden)
         self.set_policy(S.SSD_POLICY_LEDE, cand=tuple(cand or w.candidates), kmax=kmax or w.kmax,
-                        qnet_params=qp, qnet_hidden=w.qnet_hidden, fixed_k=fixed_k)
+                        qnet_params=qp, qnet_hidden=w.qnet_hidden, fixed_k=fixed_k, **sampling)
 
-    def set_threshold(self, l: int, tau: float, kmax: int):
+    def set_threshold(self, l: int, tau: float, kmax: int, **sampling):
         """Fixed exit layer l; drafting goes on while a draft's max-probability
         is >= tau (a Draft & Verify-style rule, §4.1 baselines)."""
-        self.set_policy(S.SSD_POLICY_THRESHOLD, kmax=kmax, static_l=l, conf_threshold=tau)
+        self.set_policy(S.SSD_POLICY_THRESHOLD, kmax=kmax, static_l=l, conf_threshold=tau,
+                        **sampling)
 
     # ------------------------------------------------------------ running
     def prefill(self, ids) -> int:

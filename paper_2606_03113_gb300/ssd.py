@@ -45,7 +45,8 @@ class ssd_policy(C.Structure):
                 ("static_l", C.c_int32), ("static_k", C.c_int32), ("qnet_in", C.c_int32),
                 ("qnet_hidden", C.c_int32), ("qnet_params", C.POINTER(C.c_float)),
                 ("trace_T", C.c_int32), ("topk", C.c_int32), ("fixed_k", C.c_int32),
-                ("conf_threshold", C.c_float)]
+                ("conf_threshold", C.c_float), ("temperature", C.c_float),
+                ("sample_seed", C.c_uint32)]
 
 
 class ssd_round_info(C.Structure):
@@ -63,7 +64,9 @@ class ssd_round_trace(C.Structure):
                 ("draft_margin", C.c_float * TRACE_MAXK),
                 ("verify_margin", C.c_float * (TRACE_MAXK + 1)),
                 ("verify_pmax", C.c_float * (TRACE_MAXK + 1)),
-                ("q_val", (C.c_float * 2) * TRACE_MAXQ), ("q_state", (C.c_float * 3) * TRACE_MAXQ)]
+                ("q_val", (C.c_float * 2) * TRACE_MAXQ), ("q_state", (C.c_float * 3) * TRACE_MAXQ),
+                ("sampled", C.c_int32), ("pad2", C.c_int32),
+                ("accept_margin", C.c_float * TRACE_MAXK), ("fix_margin", C.c_float)]
 
     def as_dict(self) -> dict:
         k, a, n = self.k, self.a, self.n_emit
@@ -75,7 +78,9 @@ class ssd_round_trace(C.Structure):
                     verify_margin=list(self.verify_margin[:k + 1]),
                     verify_pmax=list(self.verify_pmax[:k + 1]), q_action=list(self.q_action[:nq]),
                     q_val=[tuple(self.q_val[i]) for i in range(nq)],
-                    q_state=[tuple(self.q_state[i]) for i in range(nq)])
+                    q_state=[tuple(self.q_state[i]) for i in range(nq)],
+                    sampled=bool(self.sampled), accept_margin=list(self.accept_margin[:k]),
+                    fix_margin=self.fix_margin)
 
 
 class ssd_exit_stats(C.Structure):

@@ -51,8 +51,9 @@ def lib():
             L.synth_fill_bf16.argtypes = [u32, u32, u64, u64, dbl, p]
             L.synth_prompt.argtypes = [u32, u64, u32, p]
             L.synth_qnet_params.argtypes = [u32, ctypes.c_int, ctypes.c_int, ctypes.c_int, p]
+            L.synth_sample_uniforms.argtypes = [u32, u32, u32, u32, p]
             for f in (L.synth_philox, L.synth_fill_f32, L.synth_fill_bf16, L.synth_prompt,
-                      L.synth_qnet_params):
+                      L.synth_qnet_params, L.synth_sample_uniforms):
                 f.restype = None
             _lib = L
     return _lib
@@ -68,6 +69,14 @@ def philox4x32_10(ctr, key) -> np.ndarray:
     k = np.asarray(key, dtype=np.uint32)
     out = np.zeros(4, dtype=np.uint32)
     lib().synth_philox(_ptr(c), _ptr(k), _ptr(out))
+    return out
+
+
+def sample_uniforms(seed: int, pos: int, purpose: int, n: int) -> np.ndarray:
+    """Uniforms in (0, 1) of sampled decoding for the round at `pos`:
+    purpose 0 draws of drafts, 1 acceptance tests, 2 the round's last draw."""
+    out = np.zeros(n, dtype=np.float32)
+    lib().synth_sample_uniforms(seed, pos, purpose, n, _ptr(out))
     return out
 
 
@@ -101,7 +110,7 @@ def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
     return (b.astype(np.uint32) << 16).view(np.float32)
 
 
-__all__ = ["build", "lib", "philox4x32_10", "prompt_ids", "qnet_hidden_params", "weights_f32",
+__all__ = ["build", "lib", "philox4x32_10", "prompt_ids", "sample_uniforms", "qnet_hidden_params", "weights_f32",
            "weights_bf16_bits", "bf16_bits_to_f32", "WORKLOADS", "ModelShape", "Workload",
            "scaled_down", "SEED_WEIGHTS", "SEED_PROMPT", "SEED_QNET", "TRACE_T", "TOPK_CONF",
            "QNET_IN", "QNET_OUT", "HEADER", "TID_EMBED", "TID_LMHEAD", "layer_tid",

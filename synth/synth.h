@@ -45,6 +45,8 @@
 #define SYNTH_TID_EMBED 1u
 #define SYNTH_TID_LMHEAD 2u
 #define SYNTH_TID_QNET 3u
+/* uniforms of sampled decoding: SYNTH_TID_SAMPLE + purpose */
+#define SYNTH_TID_SAMPLE 8u
 #define SYNTH_TID_LAYER_BASE 16u
 /* per layer i: SYNTH_TID_LAYER_BASE + 4*i + one of: */
 #define SYNTH_LT_WQKV 0u
@@ -142,6 +144,16 @@ SYNTH_FN float synth_uniform_sym(uint32_t seed, uint32_t tid, uint64_t idx, doub
   int64_t a = (int64_t)(w[0] >> 8);
   double u = (double)(2 * a + 1 - 16777216) / 16777216.0;
   return (float)(u * bound);
+}
+
+/* Uniform in (0, 1) for sampled decoding: purpose (0 draw of draft i, 1
+ * acceptance test of draft i, 2 draw of the round's last token) of the round
+ * whose pending token sits at position `pos`; i < 64.  A 23-bit uniform a
+ * maps to (a + 1/2) / 2^23, exact in fp32 (24 significant bits) and fp64. */
+SYNTH_FN float synth_sample_uniform(uint32_t seed, uint32_t pos, uint32_t purpose, uint32_t i) {
+  uint32_t w[4];
+  synth_block(seed, SYNTH_TID_SAMPLE + purpose, (uint64_t)pos * 64u + i, w);
+  return ((float)(w[0] >> 9) + 0.5f) * (1.0f / 8388608.0f);
 }
 
 #endif /* SYNTH_H */

@@ -20,6 +20,10 @@ void synth_fill_bf16(uint32_t seed, uint32_t tid, uint64_t start, uint64_t n, do
     out[i] = synth_f32_to_bf16(synth_weight_f32(seed, tid, start + i, sigma_scaled));
 }
 
+void synth_sample_uniforms(uint32_t seed, uint32_t pos, uint32_t purpose, uint32_t n, float* out) {
+  for (uint32_t i = 0; i < n; ++i) out[i] = synth_sample_uniform(seed, pos, purpose, i);
+}
+
 void synth_prompt(uint32_t seed, uint64_t n, uint32_t vocab, int32_t* out) {
   for (uint64_t i = 0; i < n; ++i) out[i] = synth_token(seed, i, vocab);
 }

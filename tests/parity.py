@@ -11,6 +11,12 @@ decisions are all compared.  A round without a near-tie must match entirely
 (drafts, acceptance count, emitted tokens).  After a round with a near-tie
 the GPU restarts from the oracle's emitted sequence (ssd_resume), which
 reproduces the oracle's state (KV, trace window, pending token).
+
+Sampled decoding (temperature > 0) adds, after the verification tokens, the
+acceptance tests in the order taken (margin (p - r q) / max(p, r q); the
+kept/rejected outcome must match) and the round's last draw; a draw's margin
+(drafts and the last draw) is the distance of u S to the nearer end of the
+drawn token's CDF interval, relative to the mass S.
 """
 from __future__ import annotations
 
@@ -30,27 +36,32 @@ def has_gpu() -> bool:
 
 # Policy kinds: "ar", "static" (l, k), "lede" (cand; fixed_k > 0 drafts a
 # fixed length), "threshold" (l, tau).
-def oracle_policy(kind: str, w, qp=None, l=0, k=0, kmax=None, cand=None, fixed_k=0, tau=0.0):
+def oracle_policy(kind: str, w, qp=None, l=0, k=0, kmax=None, cand=None, fixed_k=0, tau=0.0,
+                  temperature=0.0, seed=0):
+    smp = dict(temperature=temperature, sample_seed=seed)
     if kind == "ar":
-        return oracle.make_policy(oracle.POLICY_AR)
+        return oracle.make_policy(oracle.POLICY_AR, **smp)
     if kind == "static":
-        return oracle.make_policy(oracle.POLICY_STATIC, kmax=kmax or k, static_l=l, static_k=k)
+        return oracle.make_policy(oracle.POLICY_STATIC, kmax=kmax or k, static_l=l, static_k=k,
+                                  **smp)
     if kind == "threshold":
         return oracle.make_policy(oracle.POLICY_THRESHOLD, kmax=kmax or w.kmax, static_l=l,
-                                  conf_threshold=tau)
+                                  conf_threshold=tau, **smp)
     return oracle.make_policy(oracle.POLICY_LEDE, tuple(cand or w.candidates), kmax=kmax or w.kmax,
-                              q_params=qp, q_hidden=w.qnet_hidden, fixed_k=fixed_k)
+                              q_params=qp, q_hidden=w.qnet_hidden, fixed_k=fixed_k, **smp)
 
 
-def set_gpu_policy(eng, kind: str, w, qp=None, l=0, k=0, kmax=None, cand=None, fixed_k=0, tau=0.0):
+def set_gpu_policy(eng, kind: str, w, qp=None, l=0, k=0, kmax=None, cand=None, fixed_k=0, tau=0.0,
+                   temperature=0.0, seed=0):
+    smp = dict(temperature=temperature, sample_seed=seed)
     if kind == "ar":
-        eng.set_ar()
+        eng.set_ar(**smp)
     elif kind == "static":
-        eng.set_static(l, k, kmax=kmax or k)
+        eng.set_static(l, k, kmax=kmax or k, **smp)
     elif kind == "threshold":
-        eng.set_threshold(l, tau, kmax or w.kmax)
+        eng.set_threshold(l, tau, kmax or w.kmax, **smp)
     else:
-        eng.set_lede(w, qp, kmax=kmax, cand=cand, fixed_k=fixed_k)
+        eng.set_lede(w, qp, kmax=kmax, cand=cand, fixed_k=fixed_k, **smp)
 
 
 def decision_mode(kind: str, fixed_k: int = 0) -> str:
@@ -87,25 +98,43 @@ def decisions(lg: dict, mode, thr: bool = False) -> list:
         out.append(("d", i, lg["draft_margin"][i]))
         if mode == "q" and i >= 1:
             out.append(("q", nv + i - 1, margin(nv + i - 1)))
+    if lg.get("sampled"):
+        # the verification rows' argmax decides nothing here
+        for i in range(min(lg["a"] + 1, k)):
+            out.append(("acc", i, abs(lg["accept_margin"][i])))
+        out.append(("fix", lg["a"], lg["fix_margin"]))
+        return out
     for i in range(k + 1):
         out.append(("v", i, lg["verify_margin"][i]))
     return out
 
 
 def compare_round(g: dict, lg: dict, lede, tol_tok: float, tol_q: float,
-                  q_val_tol: float, thr: bool = False):
+                  q_val_tol: float, thr: bool = False, tol_draw: float = 0.0,
+                  tol_acc: float = 0.0):
     """Compares the GPU round g with the oracle round lg decision by decision
     up to the first decision the oracle takes with a margin at or below the
     tolerance.  Returns (compared, total, clear, max Q-value error)."""
     ctx = f"round at pos {lg['pos']}: gpu {g} oracle {lg}"
     assert g["pos"] == lg["pos"] and g["x"] == lg["x"] and g["kcap"] == lg["kcap"], ctx
+    assert g.get("sampled", False) == lg.get("sampled", False), ctx
+    sampled = lg.get("sampled", False)
     ds = decisions(lg, lede, thr)
     n = 0
     q_err = 0.0
     for kind, i, margin in ds:
-        tol = tol_q if kind == "q" else tol_tok
+        tol = {"q": tol_q, "acc": tol_acc, "fix": tol_draw,
+               "d": tol_draw if sampled else tol_tok}.get(kind, tol_tok)
         if margin <= tol:
             break
+        if kind == "acc":
+            assert (g["accept_margin"][i] > 0) == (lg["accept_margin"][i] > 0), ("acc", i, ctx)
+            n += 1
+            continue
+        if kind == "fix":
+            assert g["a"] == lg["a"] and g["emitted"][i] == lg["emitted"][i], ("fix", ctx)
+            n += 1
+            continue
         if kind == "q":
             assert g["q_action"][i] == lg["q_action"][i], ("q", i, ctx)
             q_err = max(q_err, *(abs(a - b) for a, b in zip(g["q_val"][i], lg["q_val"][i])))
@@ -134,17 +163,21 @@ def first_token_margin(om, ids) -> float:
 
 def generation_parity(eng, om, w, ids, kind: str, n_new: int, tol_tok: float, tol_q: float,
                       q_val_tol: float, qp=None, l=0, k=0, kmax=None, cand=None, fixed_k=0,
-                      tau=0.0) -> dict:
+                      tau=0.0, temperature=0.0, seed=0, tol_draw=0.0, tol_acc=0.0) -> dict:
     """Returns decision counts; asserts on every compared decision."""
-    P = oracle_policy(kind, w, qp, l, k, kmax, cand, fixed_k, tau)
+    P = oracle_policy(kind, w, qp, l, k, kmax, cand, fixed_k, tau, temperature, seed)
     s = om.session(eng.max_seq)
-    ofirst = s.prefill(ids)
+    ofirst = s.prefill(ids, temperature=temperature, seed=seed)
+    first_margin = s.prefill_margin if temperature > 0 else None
     otoks, logs = s.generate(P, n_new)
-    set_gpu_policy(eng, kind, w, qp, l, k, kmax, cand, fixed_k, tau)
+    set_gpu_policy(eng, kind, w, qp, l, k, kmax, cand, fixed_k, tau, temperature, seed)
     gfirst = eng.prefill(ids)
     seq = list(ids) + [ofirst]
     if gfirst != ofirst:
-        assert first_token_margin(om, ids) <= tol_tok, (gfirst, ofirst)
+        if temperature > 0:
+            assert first_margin <= tol_draw, (gfirst, ofirst, first_margin)
+        else:
+            assert first_token_margin(om, ids) <= tol_tok, (gfirst, ofirst)
         eng.resume(seq)
     compared = total = clear_rounds = 0
     q_err = 0.0
@@ -155,7 +188,8 @@ def generation_parity(eng, om, w, ids, kind: str, n_new: int, tol_tok: float, to
         cap = n_new - done
         eng.step(cap)
         g = eng.traces(1)[0]
-        n, t, clear, qe = compare_round(g, lg, mode, tol_tok, tol_q, q_val_tol, thr)
+        n, t, clear, qe = compare_round(g, lg, mode, tol_tok, tol_q, q_val_tol, thr, tol_draw,
+                                        tol_acc)
         compared += n
         total += t
         clear_rounds += int(clear)

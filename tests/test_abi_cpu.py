@@ -71,6 +71,7 @@ def test_struct_layouts_match_header():
     assert C.sizeof(S.ssd_round_info) == 6 * 4
     t = S.ssd_round_trace
     expect = (10 + 16 + 16 + 17 + 17 + 48) * 4 + (16 + 17 + 17) * 4 + 48 * 2 * 4 + 48 * 3 * 4
+    expect += (2 + 16 + 1) * 4  # sampled, pad2, accept_margin[16], fix_margin
     assert C.sizeof(t) == expect
     assert C.sizeof(S.ssd_exit_stats) == (1 + 8 + 8 + 6) * 4
 
