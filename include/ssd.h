@@ -100,15 +100,21 @@ typedef enum {
  *             kmax (a Draft & Verify-style confidence rule with a fixed
  *             threshold).
  * kmax caps the drafts per round (1..16).  qnet_params (host fp32, copied) packs
- * W1[qnet_hidden][3], b1[qnet_hidden], W2[2][qnet_hidden], b2[2]; output 0 is
- * Q(continue), output 1 is Q(exit); ties pick continue. */
+ * W1[qnet_hidden][qnet_in], b1[qnet_hidden], W2[2][qnet_hidden], b2[2]; output
+ * 0 is Q(continue), output 1 is Q(exit); ties pick continue.  The state is
+ * the paper's s = (C_k, H, C_trace) of the exit distribution (§3.1.1) when
+ * qnet_in = 3; with qnet_in = d_model + 1 it is the pooled state: the mean,
+ * over the round's rows so far at the exit layer (the pending token in the
+ * walk; the pending token and the drafts so far while drafting), of the exit
+ * hidden state after the final RMSNorm, followed by the exit distribution's
+ * max-probability. */
 typedef struct {
   int32_t kind;
   int32_t n_cand;
   const int32_t* cand_layers;
   int32_t kmax;
   int32_t static_l, static_k;
-  int32_t qnet_in, qnet_hidden; /* qnet_in must be 3 */
+  int32_t qnet_in, qnet_hidden; /* qnet_in: 3 or d_model + 1 (state below) */
   const float* qnet_params;
   int32_t trace_T; /* C_trace window, 1..64 (paper: 20) */
   int32_t topk;    /* k of the token confidence, 1..8 (paper: 5) */

@@ -36,7 +36,9 @@ ssd_status ssd_forward_exit(ssd_ctx* ctx, const int32_t* ids, int32_t M, int32_t
                             int32_t l_exit, int32_t topk, float* logits, ssd_exit_stats* stats);
 
 /* The Q-network of the current LEDE policy on n states (host [n][3] fp32:
- * C_k, H, C_trace) -> q (host [n][2]: Q(continue), Q(exit)).  Synchronises. */
+ * C_k, H, C_trace) -> q (host [n][2]: Q(continue), Q(exit)).  SSD_ERR_STATE
+ * when the policy's network takes the pooled state (qnet_in = d_model + 1).
+ * Synchronises. */
 ssd_status ssd_qnet_eval(ssd_ctx* ctx, const float* states, int32_t n, float* q);
 
 /* KV-cache rows as fp32: layer (0-based), kind 0 = K (after RoPE) or 1 = V,

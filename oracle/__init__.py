@@ -183,14 +183,16 @@ def qnet(params: np.ndarray, hidden: int, s) -> np.ndarray:
 def make_policy(kind: int, cand=(), kmax: int = 0, static_l: int = 0, static_k: int = 0,
                 q_params: np.ndarray | None = None, q_hidden: int = 0, trace_T: int = 20,
                 topk: int = 5, fixed_k: int = 0, conf_threshold: float = 0.0,
-                temperature: float = 0.0, sample_seed: int = 0) -> Policy:
+                temperature: float = 0.0, sample_seed: int = 0, q_in: int = 3) -> Policy:
+    """q_in = 3: the paper's state (C_5, H, C_trace); q_in = d_model + 1: the
+    pooled state (mean final-normed exit state of the round's rows, pmax)."""
     P = Policy()
     P.kind = kind
     P.n_cand = len(cand)
     for i, c in enumerate(cand):
         P.cand[i] = c
     P.kmax, P.static_l, P.static_k = kmax, static_l, static_k
-    P.q_in, P.q_hidden, P.trace_T, P.topk = 3, q_hidden, trace_T, topk
+    P.q_in, P.q_hidden, P.trace_T, P.topk = q_in, q_hidden, trace_T, topk
     P.fixed_k, P.conf_threshold = fixed_k, conf_threshold
     P.temperature, P.sample_seed = temperature, sample_seed
     if q_params is not None:

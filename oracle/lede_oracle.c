@@ -540,19 +540,43 @@ double orc_trace_conf(const orc_sess* s, int T) {
   return -acc / n;
 }
 
-/* Greedy action of the Q-network on state (C_k, H, C_trace); ties choose
- * continue (= 0).  Records the decision in the round log. */
-static int q_decide(orc_sess* s, const orc_policy* P, const orc_stats* st, orc_round_log* lg) {
-  double sv[3] = {st->conf_k, st->entropy, orc_trace_conf(s, P->trace_T)};
-  double q[2];
-  orc_qnet(P->q_params, 3, P->q_hidden, sv, q);
+/* Greedy action of the Q-network; ties choose continue (= 0).  The state is
+ * the paper's (C_k, H, C_trace) (§3.1.1) when the network has 3 inputs, or,
+ * with d_model + 1 inputs, the pooled state: the mean over this round's rows
+ * so far (pool_n of them, summed in pool) of the exit hidden state after the
+ * final RMSNorm, followed by the exit distribution's max-probability.
+ * Records the decision in the round log (pooled state logged as (pmax,
+ * rows pooled, Euclidean norm of the mean)). */
+static int q_decide(orc_sess* s, const orc_policy* P, const orc_stats* st, const double* pool,
+                    int pool_n, orc_round_log* lg) {
+  const int d = s->m->c.d_model;
+  double q[2], logged[3];
+  if (P->q_in == 3) {
+    double sv[3] = {st->conf_k, st->entropy, orc_trace_conf(s, P->trace_T)};
+    orc_qnet(P->q_params, 3, P->q_hidden, sv, q);
+    for (int j = 0; j < 3; ++j) logged[j] = sv[j];
+  } else {
+    double* sv = (double*)malloc(sizeof(double) * (size_t)(d + 1));
+    if (!sv) return -1;
+    double nrm = 0.0;
+    for (int i = 0; i < d; ++i) {
+      sv[i] = pool[i] / pool_n;
+      nrm += sv[i] * sv[i];
+    }
+    sv[d] = st->pmax;
+    orc_qnet(P->q_params, d + 1, P->q_hidden, sv, q);
+    free(sv);
+    logged[0] = st->pmax;
+    logged[1] = pool_n;
+    logged[2] = sqrt(nrm);
+  }
   int a = q[1] > q[0] ? 1 : 0;
   if (lg->n_q < ORC_MAX_Q) {
     int i = lg->n_q++;
     lg->q_action[i] = a;
     lg->q_val[i][0] = q[0];
     lg->q_val[i][1] = q[1];
-    for (int j = 0; j < 3; ++j) lg->q_state[i][j] = sv[j];
+    for (int j = 0; j < 3; ++j) lg->q_state[i][j] = logged[j];
   }
   return a;
 }
@@ -661,8 +685,8 @@ static int check_policy(const orc_model* m, const orc_policy* P) {
   }
   if (P->kind != ORC_POLICY_LEDE) return ORC_ERR_ARG;
   if (P->fixed_k < 0 || P->fixed_k > ORC_MAX_K - 1) return ORC_ERR_ARG;
-  if (P->n_cand < 1 || P->n_cand > ORC_MAX_CAND || !P->q_params || P->q_in != 3 || P->q_hidden < 1 ||
-      P->trace_T < 1)
+  if (P->n_cand < 1 || P->n_cand > ORC_MAX_CAND || !P->q_params ||
+      (P->q_in != 3 && P->q_in != m->c.d_model + 1) || P->q_hidden < 1 || P->trace_T < 1)
     return ORC_ERR_ARG;
   for (int j = 0; j < P->n_cand; ++j) {
     if (P->cand[j] < 1 || P->cand[j] > L) return ORC_ERR_ARG;
@@ -813,6 +837,21 @@ int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
   double* q = NULL;
   double* pv = NULL;
   double* res = NULL;
+  /* pooled Q-network state: sum of the round's final-normed exit states */
+  const int pooled = P->kind == ORC_POLICY_LEDE && P->q_in == d + 1;
+  double* pool = NULL;
+  double* hn = NULL;
+  int pool_n = 0;
+  if (pooled) {
+    pool = (double*)malloc(sizeof(double) * (size_t)d);
+    hn = (double*)malloc(sizeof(double) * (size_t)d);
+    if (!pool || !hn) {
+      free(pool);
+      free(hn);
+      free(h);
+      return ORC_ERR_NOMEM;
+    }
+  }
   if (sampled) {
     z = (double*)malloc(sizeof(double) * (size_t)V);
     q = (double*)malloc(sizeof(double) * (size_t)(kcap > 0 ? kcap : 1) * V);
@@ -835,8 +874,16 @@ int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
       rc = orc_exit_head(m, h, z, topk, &st);
       if (rc) goto out;
       lg->visited[lg->n_visited++] = cj;
+      if (pooled) {  /* this round's rows at layer cj: the pending token only */
+        rmsnorm(h, m->final_norm, d, c->rms_eps, pool);
+        pool_n = 1;
+      }
       int act, aq = 1;
-      if (P->kind == ORC_POLICY_LEDE) aq = q_decide(s, P, &st, lg);
+      if (P->kind == ORC_POLICY_LEDE) aq = q_decide(s, P, &st, pool, pool_n, lg);
+      if (aq < 0) {
+        rc = ORC_ERR_NOMEM;
+        goto out;
+      }
       act = (j == n_c - 1) ? 1 : aq;
       if (act) {
         lstar = cj;
@@ -864,6 +911,11 @@ int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
       if (rc) goto out;
       rc = orc_exit_head(m, h, z, topk, &st);
       if (rc) goto out;
+      if (pooled) {  /* add draft row k's final-normed state at l* */
+        rmsnorm(h, m->final_norm, d, c->rms_eps, hn);
+        for (int i = 0; i < d; ++i) pool[i] += hn[i];
+        ++pool_n;
+      }
       if (sampled) {
         orc_tempered(z, V, Tmp, q + (int64_t)k * V);
         drafts[k] = orc_draw(q + (int64_t)k * V, V, uniform_of(P->sample_seed, p, 0, k),
@@ -876,9 +928,13 @@ int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
       if (P->kind == ORC_POLICY_THRESHOLD)
         keep = threshold_decide(P, &st, lg);
       else if (P->kind == ORC_POLICY_LEDE && P->fixed_k == 0)
-        keep = q_decide(s, P, &st, lg);
+        keep = q_decide(s, P, &st, pool, pool_n, lg);
       else
         keep = 1;
+      if (keep < 0) {
+        rc = ORC_ERR_NOMEM;
+        goto out;
+      }
     }
   }
   lg->k = k;
@@ -931,6 +987,8 @@ int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
   }
 out:
   free(h);
+  free(pool);
+  free(hn);
   free(z);
   free(q);
   free(pv);

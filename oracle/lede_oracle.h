@@ -56,7 +56,7 @@ typedef struct {
   int32_t cand[ORC_MAX_CAND];        /* ascending, 1..n_layers */
   int32_t kmax;
   int32_t static_l, static_k;
-  int32_t q_in, q_hidden;            /* q_in must be 3 */
+  int32_t q_in, q_hidden;            /* 3: state (C_k, H, C_trace); d_model + 1: pooled state */
   int32_t trace_T, topk;
   const float* q_params;             /* W1[h][in], b1[h], W2[2][h], b2[2] */
   int32_t fixed_k;                   /* LEDE: 0 adaptive drafting; > 0 fixed draft length */

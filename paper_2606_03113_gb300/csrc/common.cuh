@@ -36,6 +36,7 @@ struct DevPolicy {
   int32_t cand[kMaxCand];
   int32_t fixed_k;  // LEDE: fixed draft length (0: adaptive)
   float tau;        // THRESHOLD: confidence threshold on a draft's max-probability
+  int32_t q_in;     // Q-network inputs: 3 (C_k, H, C_trace) or d + 1 (pooled state)
   float temp;       // sampled decoding temperature (0: greedy)
   uint32_t seed;    // sampled decoding seed
 };
@@ -62,6 +63,7 @@ struct Ctl {
   float trace[kTraceCap];  // ring of full-model max-probabilities
   DevPolicy pol;
   float dq_zmax[kMaxDraft], dq_sum[kMaxDraft];  // sampled drafts: max logit, normaliser
+  int32_t pool_n;                                // rows in the pooled Q-network state
   ssd_round_trace cur;     // record of the round in flight
 };
 
@@ -178,6 +180,7 @@ struct Bufs {
   float2* rope;      // [max_seq][hd/2] (cos, sin)
   void* kv;          // [L][2][Hkv][max_seq][hd]
   float* qparams;    // Q-network parameters
+  float* pool;       // [d] pooled Q-network state: sum of the round's final-normed exit rows
   int32_t* out_tok;  // [max_seq] tokens emitted in the current call
   ssd_round_trace* traces;  // [max_seq]
   int32_t* pre_tok;  // [max_seq] prefill / teacher-forced token ids

@@ -263,9 +263,50 @@ __global__ void k_round_begin(Dims D, Bufs B, cudaGraphConditionalHandle draft_i
   set_cond(draft_if, kcap > 0 ? 1u : 0u);
 }
 
+// Final RMSNorm of residual row 0 (the exit hidden state of this decision's
+// row), added to the round's pool: the walk restarts the pool at each
+// candidate layer (its rows: the pending token only), a draft adds its row
+// at l*.  Every thread calls it; returns the pool's row count and leaves the
+// Euclidean norm of the pooled mean in *norm.
+template <typename T>
+__device__ int pool_exit_state(const Dims& D, const Bufs& B, const T* __restrict__ g, bool restart,
+                               int n_before, float* red, float* norm) {
+  const int tid = threadIdx.x, nw = (int)(blockDim.x >> 5);
+  const float* h = B.h;
+  float acc = 0.f;
+  for (int i = tid; i < D.d; i += blockDim.x) acc = fmaf(h[i], h[i], acc);
+  acc = warp_sum(acc);
+  if ((tid & 31) == 0) red[tid >> 5] = acc;
+  __syncthreads();
+  float ss = 0.f;
+  for (int w = 0; w < nw; ++w) ss += red[w];
+  __syncthreads();
+  const float rstd = rsqrtf(ss / (float)D.d + D.eps);
+  const int n = restart ? 1 : n_before + 1;
+  float nrm = 0.f;
+  for (int i = tid; i < D.d; i += blockDim.x) {
+    const float hn = h[i] * rstd * Elem<T>::to_f(g[i]);
+    const float v = restart ? hn : B.pool[i] + hn;
+    B.pool[i] = v;
+    const float m = v / (float)n;
+    nrm = fmaf(m, m, nrm);
+  }
+  nrm = warp_sum(nrm);
+  if ((tid & 31) == 0) red[tid >> 5] = nrm;
+  __syncthreads();
+  float t = 0.f;
+  for (int w = 0; w < nw; ++w) t += red[w];
+  __syncthreads();
+  *norm = sqrtf(t);
+  return n;
+}
+
 // Decision at a candidate exit layer (walk) or after a draft (§3.1.2, §3.3).
-// LEDE: Q = W2 relu(W1 s + b1) + b2 on s = (C_k, H, C_trace) of the exit
-// distribution in stats[0]; greedy action, ties -> continue (0).
+// LEDE: Q = W2 relu(W1 s + b1) + b2 with s = (C_k, H, C_trace) of the exit
+// distribution in stats[0] (3 inputs), or with d_model + 1 inputs the pooled
+// state: the mean over this round's rows so far of the exit hidden state
+// after the final RMSNorm, then the exit distribution's max-probability;
+// greedy action, ties -> continue (0).
 //  walk:  exit (or the last candidate, forced) fixes l* and d_1 = argmax; the
 //         action itself says whether to keep drafting; continue opens the
 //         next walk segment (next_if).
@@ -274,7 +315,9 @@ __global__ void k_round_begin(Dims D, Bufs B, cudaGraphConditionalHandle draft_i
 // Variants (Table 3, §4.1 baselines): LEDE with a fixed draft length uses the
 // Q-network only in the walk and drafts to the cap; THRESHOLD keeps drafting
 // while the draft's max-probability is >= tau (decision logged as (tau, pmax)).
+// A pooled decision is logged with state (pmax, rows pooled, |mean|).
 __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, int layer,
+                         const void* final_norm, int dtype,
                          cudaGraphConditionalHandle next_if,
                          cudaGraphConditionalHandle draft_while) {
   pdl_wait();
@@ -287,9 +330,60 @@ __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, in
   const bool lede = P.kind == SSD_POLICY_LEDE;
   const bool thr = P.kind == SSD_POLICY_THRESHOLD;
   const bool use_q = lede && (mode == kDecideWalk || P.fixed_k == 0);
+  const bool pooled = lede && P.q_in == D.d + 1;
   const int tid = threadIdx.x;
   float q0 = 0.f, q1 = 0.f;
-  if (use_q) {
+  int n_pool = 0;
+  if (pooled) {
+    const int n_before = c->pool_n;
+    float nrm = 0.f;
+    n_pool = dtype == SSD_DTYPE_BF16
+                 ? pool_exit_state(D, B, static_cast<const __nv_bfloat16*>(final_norm),
+                                   mode == kDecideWalk, n_before, red0, &nrm)
+                 : pool_exit_state(D, B, static_cast<const float*>(final_norm),
+                                   mode == kDecideWalk, n_before, red0, &nrm);
+    if (tid == 0) {
+      c->pool_n = n_pool;
+      s_state[0] = st.pmax;
+      s_state[1] = (float)n_pool;
+      s_state[2] = nrm;
+    }
+  }
+  if (use_q && pooled) {
+    // one warp per hidden unit at a time; lanes stride over the inputs
+    __syncthreads();
+    const int H = P.q_hidden, in = D.d + 1, nw = (int)(blockDim.x >> 5);
+    const int warp = tid >> 5, lane = tid & 31;
+    const float* W1 = B.qparams;
+    const float* b1 = W1 + (size_t)H * in;
+    const float* W2 = b1 + H;
+    const float* b2 = W2 + 2 * H;
+    const float pm = st.pmax, fn = (float)n_pool;
+    float a0 = 0.f, a1 = 0.f;
+    for (int j = warp; j < H; j += nw) {
+      const float* w = W1 + (size_t)j * in;
+      float z = 0.f;
+      for (int i = lane; i < D.d; i += 32) z = fmaf(w[i], B.pool[i] / fn, z);
+      z = warp_sum(z);
+      z = fmaf(w[D.d], pm, z) + b1[j];
+      const float r = fmaxf(z, 0.f);
+      a0 = fmaf(W2[j], r, a0);
+      a1 = fmaf(W2[H + j], r, a1);
+    }
+    if (lane == 0) {
+      red0[warp] = a0;
+      red1[warp] = a1;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      for (int w = 0; w < nw; ++w) {
+        q0 += red0[w];
+        q1 += red1[w];
+      }
+      q0 += b2[0];
+      q1 += b2[1];
+    }
+  } else if (use_q) {
     if (tid == 0) {
       s_state[0] = st.conf_k;
       s_state[1] = st.entropy;
@@ -646,10 +740,11 @@ cudaError_t launch_round_begin(const Dims& D, const Bufs& B, cudaGraphConditiona
 }
 
 cudaError_t launch_decide(const Dims& D, const Bufs& B, int mode, int cand_idx, int is_last,
-                          int layer, cudaGraphConditionalHandle next_if,
+                          int layer, const void* final_norm, int dtype,
+                          cudaGraphConditionalHandle next_if,
                           cudaGraphConditionalHandle draft_while, cudaStream_t st) {
   return launch_ex(k_decide, dim3(1), dim3(kSampleThreads), 0, st, D, B, mode, cand_idx, is_last,
-                   layer, next_if, draft_while);
+                   layer, final_norm, dtype, next_if, draft_while);
 }
 
 cudaError_t launch_draft_begin(const Bufs& B, cudaGraphConditionalHandle draft_while,

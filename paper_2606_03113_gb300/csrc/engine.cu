@@ -92,7 +92,9 @@ size_t layout(const ssd_model_cfg& c, char* base, Dims* D, Bufs* B) {
   b.stats = cv.take<RowStats>(sizeof(RowStats) * kMaxM);
   b.rope = cv.take<float2>(sizeof(float2) * (size_t)d.max_seq * (d.hd / 2));
   b.kv = cv.take<void>(elt * (size_t)d.L * 2 * d.Hkv * (size_t)d.max_seq * d.hd);
-  b.qparams = cv.take<float>(sizeof(float) * (6 * kMaxQHidden + 2));
+  // largest network: d + 1 inputs (pooled state), kMaxQHidden hidden units
+  b.qparams = cv.take<float>(sizeof(float) * ((size_t)kMaxQHidden * (d.d + 4) + 2));
+  b.pool = cv.take<float>(sizeof(float) * (size_t)d.d);
   b.out_tok = cv.take<int32_t>(sizeof(int32_t) * (size_t)d.max_seq);
   b.traces = cv.take<ssd_round_trace>(sizeof(ssd_round_trace) * (size_t)d.max_seq);
   b.pre_tok = cv.take<int32_t>(sizeof(int32_t) * (size_t)d.max_seq);
@@ -140,6 +142,7 @@ struct ssd_ctx {
   int kind = SSD_POLICY_AR;
   std::vector<int> cand;
   int kmax = 0, static_l = 0, static_k = 0, q_hidden = 0, trace_T = 20, topk = 5, fixed_k = 0;
+  int q_in = 3;
   bool sampled = false;  // temperature > 0: the exit heads write their logits
   // graphs
   cudaGraph_t round_g = nullptr, gen_g = nullptr;
@@ -267,7 +270,8 @@ cudaError_t build_walk(ssd_ctx* x, Seq& s, const std::vector<int>& cands, int j,
   if (j == 0) GK(launch_embed(x->D, x->B, x->cfg.dtype, x->embed, rows(kRowsWalk), false, 0, x->cap));
   GK(enqueue_layers(x, done, cands[j], rows(kRowsWalk), 1, x->cap));
   GK(enqueue_head(x, rows(kRowsWalk), 1, x->topk, x->sampled, x->cap));
-  GK(launch_decide(x->D, x->B, kDecideWalk, j, last ? 1 : 0, cands[j], next, 0, x->cap));
+  GK(launch_decide(x->D, x->B, kDecideWalk, j, last ? 1 : 0, cands[j], x->final_norm,
+                   x->cfg.dtype, next, 0, x->cap));
   GK(s.end());
   if (last) return cudaSuccess;
   cudaGraph_t body;
@@ -311,7 +315,8 @@ cudaError_t build_draft_phase(ssd_ctx* x, cudaGraph_t body) {
     GK(enqueue_layers(x, 0, cands[0], rows(kRowsDraft), 1, x->cap));
   }
   GK(enqueue_head(x, rows(kRowsDraft), 1, x->topk, x->sampled, x->cap));
-  GK(launch_decide(x->D, x->B, kDecideDraft, 0, 0, 0, 0, hw, x->cap));
+  GK(launch_decide(x->D, x->B, kDecideDraft, 0, 0, 0, x->final_norm, x->cfg.dtype, 0, hw,
+                   x->cap));
   return w.end();
 }
 
@@ -575,7 +580,8 @@ ssd_status ssd_set_policy(ssd_ctx* x, const ssd_policy* p) {
       cand.push_back(c);
       dp.cand[j] = c;
     }
-    if (p->qnet_in != 3) return fail(x, SSD_ERR_INVALID_ARG, "qnet_in must be 3");
+    if (p->qnet_in != 3 && p->qnet_in != x->cfg.d_model + 1)
+      return fail(x, SSD_ERR_INVALID_ARG, "qnet_in must be 3 or d_model + 1");
     if (p->qnet_hidden < 1 || p->qnet_hidden > kMaxQHidden || !p->qnet_params)
       return fail(x, SSD_ERR_INVALID_ARG, "qnet_hidden must be in 1..1024 with parameters");
   }
@@ -584,13 +590,15 @@ ssd_status ssd_set_policy(ssd_ctx* x, const ssd_policy* p) {
   dp.static_k = p->static_k;
   dp.n_cand = (int)cand.size();
   dp.q_hidden = p->kind == SSD_POLICY_LEDE ? p->qnet_hidden : 0;
+  dp.q_in = p->kind == SSD_POLICY_LEDE ? p->qnet_in : 3;
   dp.fixed_k = p->kind == SSD_POLICY_LEDE ? p->fixed_k : 0;
   dp.tau = p->kind == SSD_POLICY_THRESHOLD ? p->conf_threshold : 0.f;
   dp.temp = p->temperature;
   dp.seed = p->sample_seed;
   CK(x, cudaMemcpyAsync(&x->B.ctl->pol, &dp, sizeof(dp), cudaMemcpyHostToDevice, x->stream));
   if (p->kind == SSD_POLICY_LEDE)
-    CK(x, cudaMemcpyAsync(x->B.qparams, p->qnet_params, sizeof(float) * (6 * p->qnet_hidden + 2),
+    CK(x, cudaMemcpyAsync(x->B.qparams, p->qnet_params,
+                          sizeof(float) * ((size_t)p->qnet_hidden * (p->qnet_in + 3) + 2),
                           cudaMemcpyHostToDevice, x->stream));
   CK(x, cudaStreamSynchronize(x->stream));
   // The graphs depend on the policy kind, the candidate (or static) exit
@@ -608,6 +616,7 @@ ssd_status ssd_set_policy(ssd_ctx* x, const ssd_policy* p) {
   x->static_k = p->static_k;
   x->fixed_k = dp.fixed_k;
   x->q_hidden = dp.q_hidden;
+  x->q_in = dp.q_in;
   x->trace_T = dp.trace_T;
   x->topk = dp.topk;
   x->sampled = sampled;
@@ -821,6 +830,7 @@ ssd_status ssd_qnet_eval(ssd_ctx* x, const float* states, int32_t n, float* q) {
   if (!x) return fail(nullptr, SSD_ERR_INVALID_ARG, "ctx is NULL");
   if (x->kind != SSD_POLICY_LEDE || !x->have_policy)
     return fail(x, SSD_ERR_STATE, "no LEDE policy set");
+  if (x->q_in != 3) return fail(x, SSD_ERR_STATE, "the policy's Q-network does not take 3 inputs");
   const int cap = (int)std::min<size_t>(4096, (size_t)kMaxM * x->cfg.vocab / 5);
   if (!states || !q || n < 1 || n > cap) return fail(x, SSD_ERR_INVALID_ARG, "bad state batch");
   float* ds = x->B.logits;  // scratch: the logits buffer

@@ -64,7 +64,8 @@ cudaError_t launch_head(const Dims& D, const Bufs& B, int dtype, const void* lm_
 cudaError_t launch_round_begin(const Dims& D, const Bufs& B, cudaGraphConditionalHandle draft_if,
                                cudaStream_t st);
 cudaError_t launch_decide(const Dims& D, const Bufs& B, int mode, int cand_idx, int is_last,
-                          int layer, cudaGraphConditionalHandle next_if,
+                          int layer, const void* final_norm, int dtype,
+                          cudaGraphConditionalHandle next_if,
                           cudaGraphConditionalHandle draft_while, cudaStream_t st);
 cudaError_t launch_draft_begin(const Bufs& B, cudaGraphConditionalHandle draft_while,
                                cudaStream_t st);

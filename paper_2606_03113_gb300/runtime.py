@@ -102,7 +102,7 @@ class Engine:
     def set_policy(self, kind: int, cand=(), kmax: int = 0, static_l: int = 0, static_k: int = 0,
                    qnet_params: np.ndarray | None = None, qnet_hidden: int = 0, trace_T: int = 20,
                    topk: int = 5, fixed_k: int = 0, conf_threshold: float = 0.0,
-                   temperature: float = 0.0, sample_seed: int = 0):
+                   temperature: float = 0.0, sample_seed: int = 0, qnet_in: int = 3):
         """temperature > 0 turns on speculative sampling at that temperature
         (drafts drawn from the exit distribution, emitted tokens distributed
         as the full model's), with uniforms keyed by sample_seed."""
@@ -112,7 +112,7 @@ class Engine:
             self._qp = np.ascontiguousarray(qnet_params, dtype=np.float32)
             qp = self._qp.ctypes.data_as(C.POINTER(C.c_float))
         p = S.ssd_policy(kind, len(cand), C.cast(cand_arr, C.POINTER(C.c_int32)), kmax, static_l,
-                         static_k, 3, qnet_hidden, qp, trace_T, topk, fixed_k, conf_threshold,
+                         static_k, qnet_in, qnet_hidden, qp, trace_T, topk, fixed_k, conf_threshold,
                          temperature, sample_seed)
         S.ssd_set_policy(self.ctx, p)
         self.policy_kind = kind
@@ -126,12 +126,20 @@ class Engine:
         self.set_policy(S.SSD_POLICY_STATIC, kmax=kmax or k, static_l=l, static_k=k, **sampling)
 
     def set_lede(self, w: Workload, qnet_params: np.ndarray | None = None, kmax: int | None = None,
-                 cand=None, fixed_k: int = 0, **sampling):
+                 cand=None, fixed_k: int = 0, state: str = "paper", **sampling):
         """LEDE (§3.3); one candidate is the ablation without dynamic exit,
-        fixed_k > 0 the one without adaptive drafting (Table 3)."""
-        qp = qnet_params if qnet_params is not None else synth.qnet_hidden_params(3, w.qnet_hidden)
+        fixed_k > 0 the one without adaptive drafting (Table 3).  state
+        "paper": the network reads (C_5, H, C_trace); "pooled": the mean
+        final-normed exit state of the round's rows and the max-probability
+        (d_model + 1 inputs)."""
+        if state not in ("paper", "pooled"):
+            raise ValueError(f"unknown state {state!r}")
+        q_in = 3 if state == "paper" else w.shape.d_model + 1
+        qp = (qnet_params if qnet_params is not None
+              else synth.qnet_hidden_params(q_in, w.qnet_hidden))
         self.set_policy(S.SSD_POLICY_LEDE, cand=tuple(cand or w.candidates), kmax=kmax or w.kmax,
-                        qnet_params=qp, qnet_hidden=w.qnet_hidden, fixed_k=fixed_k, **sampling)
+                        qnet_params=qp, qnet_hidden=w.qnet_hidden, fixed_k=fixed_k,
+                        qnet_in=q_in, **sampling)
 
     def set_threshold(self, l: int, tau: float, kmax: int, **sampling):
         """Fixed exit layer l; drafting goes on while a draft's max-probability

@@ -39,9 +39,11 @@ def test_ssd_equals_ar_bitwise_on_gpu():
             assert np.array_equal(ar, st), (name, l, k)
         # the ablations of Table 3 and a confidence-threshold drafting rule
         qp = synth.qnet_hidden_params(3, w.qnet_hidden, seed=2)
+        qpp = synth.qnet_hidden_params(w.shape.d_model + 1, w.qnet_hidden, seed=2)
         for setp in (lambda: eng.set_lede(w, qp, fixed_k=3),
                      lambda: eng.set_lede(w, qp, cand=(w.candidates[0],)),
-                     lambda: eng.set_threshold(max(1, L // 2), 0.05, w.kmax)):
+                     lambda: eng.set_threshold(max(1, L // 2), 0.05, w.kmax),
+                     lambda: eng.set_lede(w, qpp, state="pooled")):
             setp()
             eng.prefill(ids)
             va, _, _ = eng.generate(w.gen_len)

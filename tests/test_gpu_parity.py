@@ -217,6 +217,25 @@ def test_lede_always_exit_policy_drafts_to_cap():
                     assert t["visited"] == list(w.candidates) and t["k"] == 1
 
 
+@pytest.mark.parametrize("name", ["tiny", "7b"])
+def test_pooled_state_generation_matches_oracle(name):
+    """LEDE whose Q-network reads the pooled state (the tiny configuration's
+    state: mean final-normed exit state of the round's rows, then pmax;
+    d_model + 1 inputs) under the segment-and-resync protocol."""
+    w, dm, eng, om = setup(name)
+    tol_tok, tol_q, _, q_val_tol = TOL[w.shape.dtype]
+    qp = synth.qnet_hidden_params(w.shape.d_model + 1, w.qnet_hidden, seed=2)
+    r = generation_parity(eng, om, w, prompt(w), "lede", w.gen_len, tol_tok, tol_q, q_val_tol,
+                          qp=qp, state="pooled")
+    print(name, "pooled", r)
+    need = 0.5 if w.shape.dtype == "f32" else 0.1
+    assert r["compared"] >= need * r["decisions"] and r["compared"] >= min(20, r["decisions"]), r
+    tr = eng.traces(4096)
+    assert any(t["k"] > 1 for t in tr)
+    # logged pooled state: (pmax, rows pooled, |mean|); rows = 1 in the walk
+    assert all(t["q_state"][i][1] == 1 for t in tr for i in range(len(t["visited"])))
+
+
 # --------------------------------------------- policy variants (Table 3, §4.1)
 
 
