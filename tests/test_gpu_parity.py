@@ -230,10 +230,12 @@ def test_pooled_state_generation_matches_oracle(name):
     print(name, "pooled", r)
     need = 0.5 if w.shape.dtype == "f32" else 0.1
     assert r["compared"] >= need * r["decisions"] and r["compared"] >= min(20, r["decisions"]), r
-    tr = eng.traces(4096)
-    assert any(t["k"] > 1 for t in tr)
-    # logged pooled state: (pmax, rows pooled, |mean|); rows = 1 in the walk
-    assert all(t["q_state"][i][1] == 1 for t in tr for i in range(len(t["visited"])))
+    # the last round (the protocol steps round by round): logged pooled state
+    # is (pmax, rows pooled, |mean|), one row in the walk, one more per draft
+    t = eng.traces(1)[0]
+    nv = len(t["visited"])
+    assert all(t["q_state"][i][1] == 1 for i in range(nv))
+    assert all(t["q_state"][nv + i - 1][1] == i + 1 for i in range(1, t["k"]))
 
 
 # --------------------------------------------- policy variants (Table 3, §4.1)
