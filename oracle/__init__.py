@@ -45,7 +45,7 @@ class Policy(C.Structure):
                 ("q_in", C.c_int32), ("q_hidden", C.c_int32), ("trace_T", C.c_int32),
                 ("topk", C.c_int32), ("q_params", C.c_void_p), ("fixed_k", C.c_int32),
                 ("conf_threshold", C.c_double), ("temperature", C.c_double),
-                ("sample_seed", C.c_uint32)]
+                ("sample_seed", C.c_uint32), ("discard_on_continue", C.c_int32)]
 
 
 class RoundLog(C.Structure):
@@ -183,7 +183,8 @@ def qnet(params: np.ndarray, hidden: int, s) -> np.ndarray:
 def make_policy(kind: int, cand=(), kmax: int = 0, static_l: int = 0, static_k: int = 0,
                 q_params: np.ndarray | None = None, q_hidden: int = 0, trace_T: int = 20,
                 topk: int = 5, fixed_k: int = 0, conf_threshold: float = 0.0,
-                temperature: float = 0.0, sample_seed: int = 0, q_in: int = 3) -> Policy:
+                temperature: float = 0.0, sample_seed: int = 0, q_in: int = 3,
+                discard_on_continue: bool = False) -> Policy:
     """q_in = 3: the paper's state (C_5, H, C_trace); q_in = d_model + 1: the
     pooled state (mean final-normed exit state of the round's rows, pmax)."""
     P = Policy()
@@ -195,6 +196,7 @@ def make_policy(kind: int, cand=(), kmax: int = 0, static_l: int = 0, static_k: 
     P.q_in, P.q_hidden, P.trace_T, P.topk = q_in, q_hidden, trace_T, topk
     P.fixed_k, P.conf_threshold = fixed_k, conf_threshold
     P.temperature, P.sample_seed = temperature, sample_seed
+    P.discard_on_continue = 1 if discard_on_continue else 0
     if q_params is not None:
         arr = np.ascontiguousarray(q_params, dtype=np.float32)
         P._keep = arr  # keep alive

@@ -63,6 +63,7 @@ typedef struct {
   double conf_threshold;             /* THRESHOLD: drafting goes on while pmax >= this */
   double temperature;                /* 0: greedy; > 0: speculative sampling at this temperature */
   uint32_t sample_seed;              /* key of the uniforms (synth_sample_uniform) */
+  int32_t discard_on_continue;       /* LEDE adaptive drafting: a continue drops its draft */
 } orc_policy;
 
 typedef struct {

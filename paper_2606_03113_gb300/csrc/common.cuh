@@ -35,6 +35,7 @@ struct DevPolicy {
   int32_t kind, kmax, static_l, static_k, n_cand, q_hidden, trace_T, topk;
   int32_t cand[kMaxCand];
   int32_t fixed_k;  // LEDE: fixed draft length (0: adaptive)
+  int32_t discard;  // LEDE adaptive drafting: drop a draft whose decision is continue
   float tau;        // THRESHOLD: confidence threshold on a draft's max-probability
   int32_t q_in;     // Q-network inputs: 3 (C_k, H, C_trace) or d + 1 (pooled state)
   float temp;       // sampled decoding temperature (0: greedy)

@@ -501,6 +501,12 @@ __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, in
       set_cond(draft_while, 0u);
       return;
     }
+    if (!go && use_q && P.discard) {
+      // discard reading: the continue action drops the draft it judged
+      c->keep = 0;
+      set_cond(draft_while, 0u);
+      return;
+    }
     c->tok[k + 1] = dtok;
     r.drafts[k] = dtok;
     r.draft_margin[k] = s_margin;

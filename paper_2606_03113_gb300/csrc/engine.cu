@@ -594,6 +594,7 @@ ssd_status ssd_set_policy(ssd_ctx* x, const ssd_policy* p) {
   dp.fixed_k = p->kind == SSD_POLICY_LEDE ? p->fixed_k : 0;
   dp.tau = p->kind == SSD_POLICY_THRESHOLD ? p->conf_threshold : 0.f;
   dp.temp = p->temperature;
+  dp.discard = p->kind == SSD_POLICY_LEDE && p->discard_on_continue ? 1 : 0;
   dp.seed = p->sample_seed;
   CK(x, cudaMemcpyAsync(&x->B.ctl->pol, &dp, sizeof(dp), cudaMemcpyHostToDevice, x->stream));
   if (p->kind == SSD_POLICY_LEDE)

@@ -102,7 +102,8 @@ class Engine:
     def set_policy(self, kind: int, cand=(), kmax: int = 0, static_l: int = 0, static_k: int = 0,
                    qnet_params: np.ndarray | None = None, qnet_hidden: int = 0, trace_T: int = 20,
                    topk: int = 5, fixed_k: int = 0, conf_threshold: float = 0.0,
-                   temperature: float = 0.0, sample_seed: int = 0, qnet_in: int = 3):
+                   temperature: float = 0.0, sample_seed: int = 0, qnet_in: int = 3,
+                   discard_on_continue: bool = False):
         """temperature > 0 turns on speculative sampling at that temperature
         (drafts drawn from the exit distribution, emitted tokens distributed
         as the full model's), with uniforms keyed by sample_seed."""
@@ -113,7 +114,7 @@ class Engine:
             qp = self._qp.ctypes.data_as(C.POINTER(C.c_float))
         p = S.ssd_policy(kind, len(cand), C.cast(cand_arr, C.POINTER(C.c_int32)), kmax, static_l,
                          static_k, qnet_in, qnet_hidden, qp, trace_T, topk, fixed_k, conf_threshold,
-                         temperature, sample_seed)
+                         temperature, sample_seed, 1 if discard_on_continue else 0)
         S.ssd_set_policy(self.ctx, p)
         self.policy_kind = kind
         self.kmax = 0 if kind == S.SSD_POLICY_AR else kmax
@@ -126,7 +127,8 @@ class Engine:
         self.set_policy(S.SSD_POLICY_STATIC, kmax=kmax or k, static_l=l, static_k=k, **sampling)
 
     def set_lede(self, w: Workload, qnet_params: np.ndarray | None = None, kmax: int | None = None,
-                 cand=None, fixed_k: int = 0, state: str = "paper", **sampling):
+                 cand=None, fixed_k: int = 0, state: str = "paper",
+                 discard_on_continue: bool = False, **sampling):
         """LEDE (§3.3); one candidate is the ablation without dynamic exit,
         fixed_k > 0 the one without adaptive drafting (Table 3).  state
         "paper": the network reads (C_5, H, C_trace); "pooled": the mean
@@ -139,7 +141,7 @@ class Engine:
               else synth.qnet_hidden_params(q_in, w.qnet_hidden))
         self.set_policy(S.SSD_POLICY_LEDE, cand=tuple(cand or w.candidates), kmax=kmax or w.kmax,
                         qnet_params=qp, qnet_hidden=w.qnet_hidden, fixed_k=fixed_k,
-                        qnet_in=q_in, **sampling)
+                        qnet_in=q_in, discard_on_continue=discard_on_continue, **sampling)
 
     def set_threshold(self, l: int, tau: float, kmax: int, **sampling):
         """Fixed exit layer l; drafting goes on while a draft's max-probability

@@ -46,7 +46,7 @@ class ssd_policy(C.Structure):
                 ("qnet_hidden", C.c_int32), ("qnet_params", C.POINTER(C.c_float)),
                 ("trace_T", C.c_int32), ("topk", C.c_int32), ("fixed_k", C.c_int32),
                 ("conf_threshold", C.c_float), ("temperature", C.c_float),
-                ("sample_seed", C.c_uint32)]
+                ("sample_seed", C.c_uint32), ("discard_on_continue", C.c_int32)]
 
 
 class ssd_round_info(C.Structure):

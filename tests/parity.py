@@ -37,7 +37,7 @@ def has_gpu() -> bool:
 # Policy kinds: "ar", "static" (l, k), "lede" (cand; fixed_k > 0 drafts a
 # fixed length), "threshold" (l, tau).
 def oracle_policy(kind: str, w, qp=None, l=0, k=0, kmax=None, cand=None, fixed_k=0, tau=0.0,
-                  temperature=0.0, seed=0, state="paper"):
+                  temperature=0.0, seed=0, state="paper", discard=False):
     smp = dict(temperature=temperature, sample_seed=seed)
     if kind == "ar":
         return oracle.make_policy(oracle.POLICY_AR, **smp)
@@ -50,11 +50,11 @@ def oracle_policy(kind: str, w, qp=None, l=0, k=0, kmax=None, cand=None, fixed_k
     q_in = 3 if state == "paper" else w.shape.d_model + 1
     return oracle.make_policy(oracle.POLICY_LEDE, tuple(cand or w.candidates), kmax=kmax or w.kmax,
                               q_params=qp, q_hidden=w.qnet_hidden, fixed_k=fixed_k, q_in=q_in,
-                              **smp)
+                              discard_on_continue=discard, **smp)
 
 
 def set_gpu_policy(eng, kind: str, w, qp=None, l=0, k=0, kmax=None, cand=None, fixed_k=0, tau=0.0,
-                   temperature=0.0, seed=0, state="paper"):
+                   temperature=0.0, seed=0, state="paper", discard=False):
     smp = dict(temperature=temperature, sample_seed=seed)
     if kind == "ar":
         eng.set_ar(**smp)
@@ -63,7 +63,8 @@ def set_gpu_policy(eng, kind: str, w, qp=None, l=0, k=0, kmax=None, cand=None, f
     elif kind == "threshold":
         eng.set_threshold(l, tau, kmax or w.kmax, **smp)
     else:
-        eng.set_lede(w, qp, kmax=kmax, cand=cand, fixed_k=fixed_k, state=state, **smp)
+        eng.set_lede(w, qp, kmax=kmax, cand=cand, fixed_k=fixed_k, state=state,
+                     discard_on_continue=discard, **smp)
 
 
 def decision_mode(kind: str, fixed_k: int = 0) -> str:
@@ -166,14 +167,16 @@ def first_token_margin(om, ids) -> float:
 def generation_parity(eng, om, w, ids, kind: str, n_new: int, tol_tok: float, tol_q: float,
                       q_val_tol: float, qp=None, l=0, k=0, kmax=None, cand=None, fixed_k=0,
                       tau=0.0, temperature=0.0, seed=0, tol_draw=0.0, tol_acc=0.0,
-                      state="paper") -> dict:
+                      state="paper", discard=False) -> dict:
     """Returns decision counts; asserts on every compared decision."""
-    P = oracle_policy(kind, w, qp, l, k, kmax, cand, fixed_k, tau, temperature, seed, state)
+    P = oracle_policy(kind, w, qp, l, k, kmax, cand, fixed_k, tau, temperature, seed, state,
+                      discard)
     s = om.session(eng.max_seq)
     ofirst = s.prefill(ids, temperature=temperature, seed=seed)
     first_margin = s.prefill_margin if temperature > 0 else None
     otoks, logs = s.generate(P, n_new)
-    set_gpu_policy(eng, kind, w, qp, l, k, kmax, cand, fixed_k, tau, temperature, seed, state)
+    set_gpu_policy(eng, kind, w, qp, l, k, kmax, cand, fixed_k, tau, temperature, seed, state,
+                   discard)
     gfirst = eng.prefill(ids)
     seq = list(ids) + [ofirst]
     if gfirst != ofirst:

@@ -43,7 +43,8 @@ def test_ssd_equals_ar_bitwise_on_gpu():
         for setp in (lambda: eng.set_lede(w, qp, fixed_k=3),
                      lambda: eng.set_lede(w, qp, cand=(w.candidates[0],)),
                      lambda: eng.set_threshold(max(1, L // 2), 0.05, w.kmax),
-                     lambda: eng.set_lede(w, qpp, state="pooled")):
+                     lambda: eng.set_lede(w, qpp, state="pooled"),
+                     lambda: eng.set_lede(w, qp, discard_on_continue=True)):
             setp()
             eng.prefill(ids)
             va, _, _ = eng.generate(w.gen_len)

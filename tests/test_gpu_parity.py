@@ -238,6 +238,33 @@ def test_pooled_state_generation_matches_oracle(name):
     assert all(t["q_state"][nv + i - 1][1] == i + 1 for i in range(1, t["k"]))
 
 
+def test_discard_reading_matches_oracle():
+    """The "discard" reading of adaptive drafting (a continue action drops
+    the draft it was taken on) with a pooled-state network that exits iff
+    the draft's max-probability exceeds tau: drafts are dropped in many
+    rounds, and the GPU follows the oracle decision by decision."""
+    w, dm, eng, om = setup("tiny")
+    D, tau = w.shape.d_model, 0.003
+    W1 = np.zeros((2, D + 1))
+    W1[0, D] = 1.0
+    qp = np.concatenate([W1.ravel(), [0.0, 1.0], [0.0, tau, 1.0, 0.0], [0.0, 0.0]])
+    qp = qp.astype(np.float32)
+    s = om.session(w.max_seq)
+    s.prefill(prompt(w))
+    P = oracle.make_policy(oracle.POLICY_LEDE, w.candidates, kmax=w.kmax, q_params=qp,
+                           q_hidden=2, q_in=D + 1, discard_on_continue=True)
+    _, logs = s.generate(P, w.gen_len)
+    dropped = sum(1 for lg in logs
+                  if lg["kcap"] and lg["q_action"][len(lg["visited"]):][-1:] == [0])
+    assert dropped >= 3
+    tol_tok, tol_q, _, q_val_tol = TOL[w.shape.dtype]
+    r = generation_parity(eng, om, w, prompt(w), "lede", w.gen_len, tol_tok, tol_q, q_val_tol,
+                          qp=qp, state="pooled", discard=True)
+    # the network's margin is |pmax - tau|, often below the 1e-4 Q tolerance
+    # on this flat tiny model (about 60 % of the decisions are compared)
+    assert r["compared"] >= 0.4 * r["decisions"], r
+
+
 # --------------------------------------------- policy variants (Table 3, §4.1)
 
 
@@ -251,7 +278,8 @@ def _median_exit_pmax(om, w, l):
 
 
 @pytest.mark.parametrize("name", ["tiny", "7b", "8b"])
-@pytest.mark.parametrize("variant", ["no_dynamic_exit", "no_adaptive_drafting", "threshold"])
+@pytest.mark.parametrize("variant", ["no_dynamic_exit", "no_adaptive_drafting", "threshold",
+                                     "discard_on_continue"])
 def test_policy_variants_match_oracle(name, variant):
     """The ablations of Table 3 (a single candidate exit layer; a fixed draft
     length after the walk) and a Draft & Verify-style confidence threshold
@@ -265,6 +293,8 @@ def test_policy_variants_match_oracle(name, variant):
         kind, kw = "lede", dict(cand=(w.candidates[len(w.candidates) // 2],))
     elif variant == "no_adaptive_drafting":
         kind, kw = "lede", dict(fixed_k=min(4, w.kmax))
+    elif variant == "discard_on_continue":
+        kind, kw = "lede", dict(discard=True)
     else:
         l = max(1, L // 2)
         kind, kw = "threshold", dict(l=l, tau=_median_exit_pmax(om, w, l))

@@ -11,7 +11,10 @@ inputs), against a numpy restatement and hand-set networks:
   pending token at each walk candidate, the pending token and the drafts so
   far at l* while drafting;
 - greedy self-speculative decoding with the pooled state still emits the
-  autoregressive tokens.
+  autoregressive tokens;
+- the "discard" reading of adaptive drafting (a continue action drops the
+  draft it was taken on), against the default "keep" reading, on a network
+  whose decisions are known from the logged max-probabilities.
 """
 import numpy as np
 import pytest
@@ -129,3 +132,44 @@ def test_pooled_state_rejects_other_widths(om):
                            q_in=D)
     with pytest.raises(oracle.OracleError):
         s.round(P, 8)
+
+
+# ------------------------------------------------- the "discard" reading
+
+
+@pytest.mark.parametrize("discard", [False, True])
+def test_discard_reading_of_adaptive_drafting(om, discard):
+    """With a network that exits iff pmax > tau, the keep reading (default)
+    keeps every draft and stops after the first continue; the discard
+    reading drops the draft whose decision was continue.  Either way the
+    output is the autoregressive one."""
+    tau = 0.003
+    W1 = np.zeros((2, D + 1))
+    W1[0, D] = 1.0
+    b1 = np.array([0.0, 1.0])
+    W2 = np.array([[0.0, tau], [1.0, 0.0]])
+    qp = _pack(W1, b1, W2, np.zeros(2))
+    ids = synth.prompt_ids(W.prompt_len, S.vocab)
+    s = om.session(W.max_seq)
+    s.prefill(ids)
+    ar, _ = s.generate(oracle.make_policy(oracle.POLICY_AR), W.gen_len)
+    s.prefill(ids)
+    P = oracle.make_policy(oracle.POLICY_LEDE, W.candidates, kmax=4, q_params=qp, q_hidden=2,
+                           q_in=D + 1, discard_on_continue=discard)
+    out, logs = s.generate(P, W.gen_len)
+    assert np.array_equal(ar, out)
+    dropped = 0
+    for lg in logs:
+        if lg["kcap"] == 0:
+            continue
+        nv = len(lg["visited"])
+        after = lg["q_action"][nv:]  # decisions taken on drafts 2, 3, ...
+        assert all(after[:-1])  # drafting goes on while the action is exit
+        stop = len(after) > 0 and after[-1] == 0
+        if discard and stop:
+            assert lg["k"] == len(after)  # d_1 and the drafts whose action was exit
+            dropped += 1
+        else:
+            assert lg["k"] == 1 + len(after)
+    if discard:
+        assert dropped >= 3
