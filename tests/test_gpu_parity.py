@@ -244,15 +244,15 @@ def test_discard_reading_matches_oracle():
     the draft's max-probability exceeds tau: drafts are dropped in many
     rounds, and the GPU follows the oracle decision by decision."""
     w, dm, eng, om = setup("tiny")
-    D, tau = w.shape.d_model, 0.003
-    W1 = np.zeros((2, D + 1))
-    W1[0, D] = 1.0
-    qp = np.concatenate([W1.ravel(), [0.0, 1.0], [0.0, tau, 1.0, 0.0], [0.0, 0.0]])
-    qp = qp.astype(np.float32)
+    D, H, tau = w.shape.d_model, w.qnet_hidden, 0.003
+    # unit 0 = pmax, unit 1 = 1; Q(continue) = tau, Q(exit) = pmax
+    W1, b1, W2 = np.zeros((H, D + 1)), np.zeros(H), np.zeros((2, H))
+    W1[0, D], b1[1], W2[0, 1], W2[1, 0] = 1.0, 1.0, tau, 1.0
+    qp = np.concatenate([W1.ravel(), b1, W2.ravel(), np.zeros(2)]).astype(np.float32)
     s = om.session(w.max_seq)
     s.prefill(prompt(w))
     P = oracle.make_policy(oracle.POLICY_LEDE, w.candidates, kmax=w.kmax, q_params=qp,
-                           q_hidden=2, q_in=D + 1, discard_on_continue=True)
+                           q_hidden=H, q_in=D + 1, discard_on_continue=True)
     _, logs = s.generate(P, w.gen_len)
     dropped = sum(1 for lg in logs
                   if lg["kcap"] and lg["q_action"][len(lg["visited"]):][-1:] == [0])
