@@ -86,7 +86,8 @@ typedef enum {
 } ssd_policy_kind;
 
 /* Speculation policy (§3.3 and the baselines and ablations of §4.1, Table 3).
- *  AR:        plain greedy decoding with the full model (one token per round).
+ *  AR:        plain decoding with the full model (one token per round; greedy,
+ *             or drawn at the policy's temperature).
  *  STATIC:    fixed exit layer static_l and draft length static_k (LayerSkip).
  *  LEDE:      Q-network over candidate exit layers cand_layers[0..n_cand),
  *             ascending in 1..n_layers; forced exit at the last one; adaptive

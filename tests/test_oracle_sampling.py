@@ -14,7 +14,9 @@ oracle itself:
   for the emitted tokens, so the test has power;
 - at l* = L the draft and target distributions coincide and every draft is
   kept;
-- as the temperature goes to 0 the sampled rounds emit the greedy tokens.
+- as the temperature goes to 0 the sampled rounds emit the greedy tokens;
+- autoregressive sampling equals numpy's inverse CDF of scipy's softmax at
+  the uniforms keyed by position (independent forward passes per token).
 """
 import numpy as np
 import pytest
@@ -217,3 +219,31 @@ def test_sampled_prefill_draws_from_full_model(micro):
     stat, crit = _chi2(counts, p, N)
     assert stat < crit, (stat, crit)
     assert s.prefill(ids) == int(np.argmax(z))
+
+
+def test_ar_sampling_equals_numpy_restatement(micro):
+    """Autoregressive decoding at T = 0.7: every token is numpy's inverse
+    CDF (searchsorted over the cumulative sum of scipy's softmax(z / T)) at
+    the uniform keyed by (seed, position of the row's input token, purpose
+    2, index 0), with z from an independent full-prefix forward pass; the
+    token after the prompt uses the key of the last prompt position."""
+    from scipy.special import softmax
+    om, s = micro
+    T, seed, n = 0.7, 21, 24
+    ids = list(synth.prompt_ids(8, MICRO.vocab))
+    first = s.prefill(ids, temperature=T, seed=seed)
+    out, logs = s.generate(oracle.make_policy(oracle.POLICY_AR, temperature=T, sample_seed=seed), n)
+    toks = [first] + [int(t) for t in out]
+    seq = ids + toks
+    checked = 0
+    for j, tok in enumerate(toks):
+        pre = seq[:len(ids) + j]  # the row that chose tok reads pre[-1]
+        z, _ = om.exit_head(s.forward(pre, 0, 0, MICRO.n_layers)[-1])
+        C = np.cumsum(softmax(z / T))
+        u = float(synth.sample_uniforms(seed, len(pre) - 1, 2, 1)[0])
+        ref = int(np.searchsorted(C, u * C[-1], side="right"))
+        lo = C[ref - 1] if ref else 0.0
+        if min(u * C[-1] - lo, C[ref] - u * C[-1]) > 1e-9:
+            assert tok == ref, j
+            checked += 1
+    assert len(logs) == n and checked >= n - 2
