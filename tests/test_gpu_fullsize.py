@@ -13,7 +13,8 @@ size:
 - greedy self-speculative decoding after the workload's full prompt emits
   exactly the autoregressive tokens, for the seeded LEDE Q-network and for a
   static (L/2, 4) policy (§3.3 with greedy acceptance, §4.1);
-- exiting at l = L accepts every draft (shared exit head, §3.1.1);
+- exiting at l = L accepts every draft (shared exit head, §3.1.1), greedy
+  and with speculative sampling at temperature 0.6;
 - Llama-2-7B shape (the benchmark's workload): teacher-forced logits at the
   exits l = L/2 and l = L within 2e-2 max relative error of the oracle's
   full model on a short prompt.
@@ -156,14 +157,19 @@ def test_ssd_equals_ar_after_full_prompt(full):
     assert np.array_equal(ar, st), name
 
 
-def test_full_depth_exit_accepts_every_draft(full):
+@pytest.mark.parametrize("temperature", [0.0, 0.6])
+def test_full_depth_exit_accepts_every_draft(full, temperature):
+    """Greedy: every draft equals the verification argmax.  Sampled (the
+    acceptance rule of §4.1 over the full vocabulary): the draft and target
+    distributions coincide, so every acceptance test keeps its draft."""
     name, w, dm, eng = full
     L = w.shape.n_layers
-    eng.set_static(L, 4, kmax=4)
+    eng.set_static(L, 4, kmax=4, temperature=temperature, sample_seed=4)
     eng.prefill(prompt(w))
     _, nr, _ = eng.generate(min(40, GEN[name]))
     tr = eng.traces(nr)
     assert all(t["a"] == t["k"] and t["lstar"] == L for t in tr if t["kcap"] > 0)
+    assert all(t["sampled"] == (temperature > 0) for t in tr)
 
 
 def test_teacher_forced_logits_full_7b(full):
