@@ -1,0 +1,93 @@
+"""Host logic of bench.py on the CPU: the algorithmic bytes of a round, the
+kernel-launch count of a round graph, the ncu traffic lookup and the clock
+record parser."""
+import os
+import re
+import sys
+
+import pytest
+
+REPO = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, REPO)
+
+import bench  # noqa: E402
+from paper_2606_03113_gb300.runtime import kernels_per_round, pass_launches  # noqa: E402
+from synth.workloads import LLAMA2_7B, TINY  # noqa: E402
+
+
+def test_round_bytes_worked_example():
+    """Llama-2-7B shape, two candidates visited, exit at layer 8, six drafts,
+    context about 640: 2 LM heads + 6 partial passes of 8 layers (5 with a
+    head) + one full pass with a head, plus the KV of each pass, about
+    35.3 GB per round."""
+    s = LLAMA2_7B.shape
+    tr = dict(pos=637, kcap=12, visited=[4, 8], lstar=8, k=6)
+    b = bench.round_bytes(LLAMA2_7B, tr)
+    Wl, head = s.layer_weight_bytes(), s.lm_head_bytes()
+    assert Wl == 404750336 and head == 262144000
+    weights = 2 * head + 6 * 8 * Wl + 5 * head + 32 * Wl + head
+    assert weights < b < weights + 1.0e9  # KV: 16 KB per position and layer
+    assert b == pytest.approx(35.3e9, rel=0.01)
+
+
+def test_round_bytes_autoregressive():
+    s = LLAMA2_7B.shape
+    pos = 700
+    tr = dict(pos=pos, kcap=0, visited=[], lstar=0, k=0)
+    kv = 2 * s.n_kv_heads * s.head_dim * 2 * (pos + 1)  # K and V rows read per layer
+    assert bench.round_bytes(LLAMA2_7B, tr) == s.n_layers * (s.layer_weight_bytes() + kv) \
+        + s.lm_head_bytes()
+
+
+def test_kernel_launches_of_a_round():
+    L = LLAMA2_7B.shape.n_layers
+    # bf16 pass over n layers: first QKV, then attention + chained launch per layer
+    assert [pass_launches(n) for n in (0, 1, 4)] == [0, 3, 9]
+    assert pass_launches(4, bf16=False) == 20
+    # autoregressive round: round_begin, embed, pass, head, accept
+    ar = dict(kcap=0, visited=[], lstar=0, k=0)
+    assert kernels_per_round(ar, L, 0) == 1 + 1 + (2 * L + 1) + 1 + 1
+    # LEDE round: walk over candidates 4 and 8 (segment pass, head, decide),
+    # draft_begin, two further drafts (embed, 8 layers, head, decide), verify
+    tr = dict(kcap=12, visited=[4, 8], lstar=8, k=3)
+    walk = 1 + (9 + 2) + (9 + 2)
+    drafts = 1 + 2 * (1 + 17 + 2)
+    verify = 1 + (2 * L + 1) + 1 + 1
+    assert kernels_per_round(tr, L, 0) == 1 + walk + drafts + verify
+    assert bench.kernels_in_round(LLAMA2_7B, tr) == 1 + walk + drafts + verify
+    assert bench.kernels_in_round(TINY, ar) == 1 + 1 + 5 * TINY.shape.n_layers + 1 + 1
+
+
+def test_measured_traffic_follows_the_profile_hash(tmp_path, monkeypatch):
+    v = bench.measured_traffic("k_chain(o+gate_up+down+next_qkv)")
+    assert v is None or v == 414328320
+    assert bench.measured_traffic("k_attn") is None  # no traffic summary for it
+    # a profile whose recorded hash differs from the sources gives no number
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    text = open(os.path.join(REPO, "profiles", "k_chain_llama2-7b.md")).read()
+    digest = re.search(r"`([0-9a-f]{64})`", text).group(1)
+    other = ("0" if digest[0] != "0" else "1") + digest[1:]
+    (prof / "k_chain_llama2-7b.md").write_text(text.replace(digest, other))
+    csrc = tmp_path / "paper_2606_03113_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    for f in bench.TRAFFIC_SOURCES:
+        (csrc / f).write_bytes(open(os.path.join(REPO, "paper_2606_03113_gb300", "csrc", f),
+                                    "rb").read())
+    monkeypatch.setattr(bench, "REPO", str(tmp_path))
+    assert bench.measured_traffic("k_chain(o+gate_up+down+next_qkv)") is None
+
+
+def test_clock_record_parser(tmp_path):
+    path = tmp_path / "clocks.csv"
+    rows = ["0, 2070, 2070, 900.1, 0x0, Not Active, Not Active, Not Active, Not Active",
+            "0, 2055, 2070, 950.0, 0x4, Not Active, Not Active, Not Active, Active",
+            "0, 2070, 2070, 960.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+            "garbage line"]
+    path.write_text("\n".join(rows) + "\n")
+    cs = bench.ClockSampler(0)
+    cs.path = str(path)
+    out = cs.summary()
+    assert out["sm_mhz"] == 2070.0 and out["sm_max_mhz"] == 2070.0
+    assert out["reasons"] == ["sw_power_cap"] and out["samples"] == 3
+    assert not path.exists()  # the record is removed after reading
