@@ -6,7 +6,9 @@ acceptance count is what independent full-prefix passes give).
 Each hand-built case is chosen so that a plausible mistake fails it: the RoPE
 pairing and sign, the attention scale, the GQA head mapping, the gate/up
 order of SwiGLU, the norm epsilon and weight, the Q-network layout and its tie
-rule, the forced exit, and the round's acceptance/rollback bookkeeping.
+rule, the forced exit, and the round's acceptance/rollback bookkeeping.  On
+the tiny configuration itself, the oracle's logits at exits 1, 2 and 4 equal a
+numpy restatement of the whole decoder within 1e-9.
 """
 import math
 
@@ -469,3 +471,73 @@ def test_variant_policies_rejected_when_malformed(tiny_setup):
     for P in bad:
         with pytest.raises(oracle.OracleError):
             s.round(P, 10)
+
+
+# ------------------------------------------------ composition on a real shape
+
+
+def _numpy_forward(shape, ids, l_exit):
+    """The Llama decoder of the tiny configuration written out in numpy
+    (weights from the seeded generator): pre-RMSNorm blocks with RoPE
+    ("rotate half", angle pos * theta^(-2i/hd)), causal GQA attention scaled
+    by 1/sqrt(hd), SwiGLU down(silu(gate) * up), the second half's out/down
+    projections scaled; then the shared final RMSNorm and LM head on the
+    hidden states after l_exit blocks.  Returns logits [n][vocab]."""
+    s = shape
+    d, hd, Hq, Hkv, F, V = s.d_model, s.head_dim, s.n_heads, s.n_kv_heads, s.ffn_dim, s.vocab
+
+    def mat(tid, rows, cols, sig):
+        return synth.weights_f32(synth.SEED_WEIGHTS, tid, 0, rows * cols, sig).astype(
+            np.float64).reshape(rows, cols)
+
+    def rms(x):
+        return x / np.sqrt((x * x).mean(axis=-1, keepdims=True) + s.rms_eps)
+
+    n = len(ids)
+    pos = np.arange(n)[:, None]
+    ang = pos * s.rope_theta ** (-2.0 * np.arange(hd // 2) / hd)[None, :]
+    cos, sin = np.cos(ang), np.sin(ang)
+
+    def rope(v):  # v [n][heads][hd]
+        a, b = v[..., :hd // 2], v[..., hd // 2:]
+        c, si = cos[:, None, :], sin[:, None, :]
+        return np.concatenate([a * c - b * si, a * si + b * c], axis=-1)
+
+    h = mat(synth.TID_EMBED, V, d, s.sigma)[ids]
+    for l in range(l_exit):
+        late = s.late_scale if l >= s.n_layers // 2 else 1.0
+        wqkv = mat(synth.layer_tid(l, 0), (Hq + 2 * Hkv) * hd, d, s.sigma)
+        wo = mat(synth.layer_tid(l, 1), d, Hq * hd, s.sigma * late)
+        wgu = mat(synth.layer_tid(l, 2), 2 * F, d, s.sigma)
+        wdown = mat(synth.layer_tid(l, 3), d, F, s.sigma * late)
+        qkv = rms(h) @ wqkv.T
+        q = rope(qkv[:, :Hq * hd].reshape(n, Hq, hd))
+        k = rope(qkv[:, Hq * hd:(Hq + Hkv) * hd].reshape(n, Hkv, hd))
+        v = qkv[:, (Hq + Hkv) * hd:].reshape(n, Hkv, hd)
+        out = np.zeros((n, Hq, hd))
+        for hq in range(Hq):
+            kv = hq // (Hq // Hkv)
+            sc = q[:, hq, :] @ k[:, kv, :].T / math.sqrt(hd)
+            sc = np.where(np.tril(np.ones((n, n))) > 0, sc, -np.inf)
+            p = np.exp(sc - sc.max(axis=1, keepdims=True))
+            out[:, hq, :] = (p / p.sum(axis=1, keepdims=True)) @ v[:, kv, :]
+        h = h + out.reshape(n, Hq * hd) @ wo.T
+        gu = rms(h) @ wgu.T
+        g, u = gu[:, :F], gu[:, F:]
+        h = h + (g / (1.0 + np.exp(-g)) * u) @ wdown.T
+    return rms(h) @ mat(synth.TID_LMHEAD, V, d, s.sigma).T
+
+
+@pytest.mark.parametrize("l_exit", [1, 2, 4])
+def test_numpy_restatement_of_the_tiny_forward(l_exit):
+    s = TINY.shape
+    ids = list(synth.prompt_ids(12, s.vocab))
+    ref = _numpy_forward(s, ids, l_exit)
+    om = oracle.Model(s)
+    try:
+        h = om.session(32).forward(ids, 0, 0, l_exit)
+        for i in range(len(ids)):
+            z = om.logits(h[i])
+            assert np.abs(z - ref[i]).max() <= 1e-9 * np.abs(ref[i]).max(), (l_exit, i)
+    finally:
+        om.close()
