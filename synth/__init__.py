@@ -110,8 +110,8 @@ def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
     return (b.astype(np.uint32) << 16).view(np.float32)
 
 
-__all__ = ["build", "lib", "philox4x32_10", "prompt_ids", "sample_uniforms", "qnet_hidden_params", "weights_f32",
-           "weights_bf16_bits", "bf16_bits_to_f32", "WORKLOADS", "ModelShape", "Workload",
+__all__ = ["build", "lib", "philox4x32_10", "prompt_ids", "sample_uniforms", "qnet_hidden_params",
+           "weights_f32", "weights_bf16_bits", "bf16_bits_to_f32", "WORKLOADS", "ModelShape", "Workload",
            "scaled_down", "SEED_WEIGHTS", "SEED_PROMPT", "SEED_QNET", "TRACE_T", "TOPK_CONF",
            "QNET_IN", "QNET_OUT", "HEADER", "TID_EMBED", "TID_LMHEAD", "layer_tid",
            "LT_WQKV", "LT_WO", "LT_WGU", "LT_WDOWN"]

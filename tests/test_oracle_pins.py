@@ -8,7 +8,8 @@ pairing and sign, the attention scale, the GQA head mapping, the gate/up
 order of SwiGLU, the norm epsilon and weight, the Q-network layout and its tie
 rule, the forced exit, and the round's acceptance/rollback bookkeeping.  On
 the tiny configuration itself, the oracle's logits at exits 1, 2 and 4 equal a
-numpy restatement of the whole decoder within 1e-9.
+numpy restatement of the whole decoder within 1e-9 (and on a bf16
+grouped-query member of the Llama-3 family).
 """
 import math
 
@@ -487,8 +488,12 @@ def _numpy_forward(shape, ids, l_exit):
     d, hd, Hq, Hkv, F, V = s.d_model, s.head_dim, s.n_heads, s.n_kv_heads, s.ffn_dim, s.vocab
 
     def mat(tid, rows, cols, sig):
-        return synth.weights_f32(synth.SEED_WEIGHTS, tid, 0, rows * cols, sig).astype(
-            np.float64).reshape(rows, cols)
+        if s.dtype == "bf16":  # bf16 storage: the generator's values rounded to bf16
+            w = synth.bf16_bits_to_f32(
+                synth.weights_bf16_bits(synth.SEED_WEIGHTS, tid, 0, rows * cols, sig))
+        else:
+            w = synth.weights_f32(synth.SEED_WEIGHTS, tid, 0, rows * cols, sig)
+        return w.astype(np.float64).reshape(rows, cols)
 
     def rms(x):
         return x / np.sqrt((x * x).mean(axis=-1, keepdims=True) + s.rms_eps)
@@ -528,9 +533,16 @@ def _numpy_forward(shape, ids, l_exit):
     return rms(h) @ mat(synth.TID_LMHEAD, V, d, s.sigma).T
 
 
-@pytest.mark.parametrize("l_exit", [1, 2, 4])
-def test_numpy_restatement_of_the_tiny_forward(l_exit):
-    s = TINY.shape
+# a bf16 member of the Llama-3 family: grouped-query attention (4 query heads
+# per KV head), theta 500000, bf16 weights and embeddings
+SMALL_GQA_BF16 = ModelShape("gqa-bf16", 4, 256, 8, 2, 32, 512, 1024, 1e-5, 500000.0, "bf16",
+                            sigma=0.05, late_scale=0.2)
+
+
+@pytest.mark.parametrize("shape,l_exit", [(TINY.shape, 1), (TINY.shape, 2), (TINY.shape, 4),
+                                          (SMALL_GQA_BF16, 3), (SMALL_GQA_BF16, 4)])
+def test_numpy_restatement_of_the_tiny_forward(shape, l_exit):
+    s = shape
     ids = list(synth.prompt_ids(12, s.vocab))
     ref = _numpy_forward(s, ids, l_exit)
     om = oracle.Model(s)
