@@ -84,3 +84,30 @@ def test_product_path_has_no_oracle_import():
                 src = open(os.path.join(root, f)).read()
                 assert "import oracle" not in src and "from oracle" not in src, f
                 assert "lede_oracle" not in src, f
+
+
+def test_struct_layouts_match_the_c_compiler(tmp_path):
+    """Every field of every struct the binding mirrors sits at the offset the
+    C compiler gives it from include/ssd.h and include/ssd_ops.h."""
+    import subprocess
+    structs = [S.ssd_model_cfg, S.ssd_weights, S.ssd_policy, S.ssd_round_info,
+               S.ssd_round_trace, S.ssd_exit_stats]
+    lines = ['#include <stdio.h>', '#include "ssd_ops.h"', "int main(void) {"]
+    for st in structs:
+        name = st.__name__
+        lines.append(f'  printf("{name} sizeof %zu\\n", sizeof({name}));')
+        for field, _ in st._fields_:
+            lines.append(f'  printf("{name} {field} %zu\\n", offsetof({name}, {field}));')
+    lines += ["  return 0;", "}"]
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    subprocess.check_call(["gcc", "-std=c11", "-I", inc, str(src), "-o", str(exe)])
+    out = subprocess.check_output([str(exe)], text=True).split("\n")
+    got = {tuple(l.split()[:2]): int(l.split()[2]) for l in out if l.strip()}
+    for st in structs:
+        name = st.__name__
+        assert got[(name, "sizeof")] == C.sizeof(st), name
+        for field, _ in st._fields_:
+            assert got[(name, field)] == getattr(st, field).offset, (name, field)

@@ -553,3 +553,31 @@ def test_numpy_restatement_of_the_tiny_forward(shape, l_exit):
             assert np.abs(z - ref[i]).max() <= 1e-9 * np.abs(ref[i]).max(), (l_exit, i)
     finally:
         om.close()
+
+
+def test_oracle_struct_layouts_match_the_c_compiler(tmp_path):
+    """The ctypes mirrors of the oracle's structs match lede_oracle.h field
+    by field (a mismatch would silently corrupt every oracle result)."""
+    import ctypes
+    import os
+    import subprocess
+    structs = {"orc_cfg": oracle.Cfg, "orc_stats": oracle.Stats, "orc_policy": oracle.Policy,
+               "orc_round_log": oracle.RoundLog}
+    lines = ['#include <stddef.h>', '#include <stdio.h>', '#include "lede_oracle.h"',
+             "int main(void) {"]
+    for cname, st in structs.items():
+        lines.append(f'  printf("{cname} sizeof %zu\\n", sizeof({cname}));')
+        for field, _ in st._fields_:
+            lines.append(f'  printf("{cname} {field} %zu\\n", offsetof({cname}, {field}));')
+    lines += ["  return 0;", "}"]
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    subprocess.check_call(["gcc", "-std=c11", "-I", os.path.dirname(oracle.__file__), str(src),
+                           "-o", str(exe)])
+    out = subprocess.check_output([str(exe)], text=True).split("\n")
+    got = {tuple(l.split()[:2]): int(l.split()[2]) for l in out if l.strip()}
+    for cname, st in structs.items():
+        assert got[(cname, "sizeof")] == ctypes.sizeof(st), cname
+        for field, _ in st._fields_:
+            assert got[(cname, field)] == getattr(st, field).offset, (cname, field)
