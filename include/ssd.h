@@ -130,7 +130,7 @@ typedef struct {
   uint32_t sample_seed;
   /* LEDE adaptive drafting: 0 (default) keeps each draft and lets the
    * decision on its state say whether to draft another; 1 drops a draft
-   * whose decision is continue (the action judges the draft it was taken
+   * whose decision is continue (the action is about the draft it was taken
    * on) and stops drafting.  The walk's exit always keeps d_1. */
   int32_t discard_on_continue;
 } ssd_policy;

@@ -936,7 +936,7 @@ int orc_round(orc_sess* s, const orc_policy* P, int cap, orc_round_log* lg) {
         goto out;
       }
       /* the "discard" reading of adaptive drafting: the continue action
-       * judges the draft it was taken on, which is dropped */
+       * is about the draft it was taken on, which is dropped */
       if (!keep && P->kind == ORC_POLICY_LEDE && P->fixed_k == 0 && P->discard_on_continue) --k;
     }
   }

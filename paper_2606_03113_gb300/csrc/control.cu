@@ -502,7 +502,7 @@ __global__ void k_decide(Dims D, Bufs B, int mode, int cand_idx, int is_last, in
       return;
     }
     if (!go && use_q && P.discard) {
-      // discard reading: the continue action drops the draft it judged
+      // discard reading: the continue action drops the draft it was taken on
       c->keep = 0;
       set_cond(draft_while, 0u);
       return;
