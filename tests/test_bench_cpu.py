@@ -91,3 +91,24 @@ def test_clock_record_parser(tmp_path):
     assert out["sm_mhz"] == 2070.0 and out["sm_max_mhz"] == 2070.0
     assert out["reasons"] == ["sw_power_cap"] and out["samples"] == 3
     assert not path.exists()  # the record is removed after reading
+
+
+def test_reference_arm_prints_the_contract_line():
+    """`bench.py --impl reference` times the oracle on the host cores and
+    prints one JSON line with the contract's keys (tiny workload here)."""
+    import json
+    import subprocess
+    out = subprocess.check_output(
+        [sys.executable, os.path.join(REPO, "bench.py"), "--impl", "reference", "--workload",
+         "tiny", "--steps", "1", "--warmup", "0"], text=True, timeout=300, cwd=REPO)
+    lines = [l for l in out.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+                "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config"):
+        assert key in d, key
+    assert d["impl"] == "reference" and d["value"] > 0 and d["higher_is_better"] is True
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
+    assert d["cpu_baseline"]["value"] == d["value"]
+    assert d["e2e"] == dict(value=d["value"], unit=d["unit"], h2d_bytes_per_step=0,
+                            d2h_bytes_per_step=0)
