@@ -321,6 +321,8 @@ def main():
     ap.add_argument("--train-prompts", type=int, default=4)
     ap.add_argument("--train-gen", type=int, default=128)
     ap.add_argument("--train-episodes", type=int, default=30000)
+    ap.add_argument("--save-exit-table", default="",
+                    help="write the Q-network's training experience to this .npz file")
     ap.add_argument("--gen", type=int, default=0, help="new tokens per step (default: workload)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-compare", action="store_true", help="skip the AR / static lines")
@@ -377,6 +379,8 @@ def main():
         prompts = [synth.prompt_ids(128, w.shape.vocab, seed=synth.SEED_PROMPT + 1 + i)
                    for i in range(args.train_prompts)]
         table = PL.collect_exit_table(eng, w.candidates, prompts, args.train_gen)
+        if args.save_exit_table and rank == 0:
+            table.save(args.save_exit_table)
         t1 = time.perf_counter()
         qp, walk, tlog = PL.train_policy(table, w.qnet_hidden, episodes=args.train_episodes)
         t2 = time.perf_counter()

@@ -77,6 +77,17 @@ class ExitTable:
         per candidate layer."""
         return self.correct.mean(axis=0)
 
+    def save(self, path: str):
+        """Writes the table (not the token sequences) as a .npz file."""
+        np.savez(path, cands=np.asarray(self.cands), n_layers=self.n_layers, conf=self.conf,
+                 ent=self.ent, trace=self.trace, correct=self.correct)
+
+    @staticmethod
+    def load(path: str) -> "ExitTable":
+        z = np.load(path)
+        return ExitTable(tuple(int(c) for c in z["cands"]), int(z["n_layers"]), z["conf"],
+                         z["ent"], z["trace"], z["correct"].astype(bool))
+
 
 def _trace_conf(pmax_hist) -> float:
     h = list(pmax_hist)[-TRACE_T:]

@@ -62,3 +62,17 @@ def test_export_layout_matches_the_oracle_qnet():
         q_ref = net.q(s[None, :], noisy=False)[0]
         q_orc = oracle.qnet(params, 16, s)
         assert np.allclose(q_orc, q_ref, rtol=1e-4, atol=1e-4)
+
+
+def test_exit_table_save_and_load_round_trip(tmp_path):
+    from paper_2606_03113_gb300.policy import ExitTable
+    rng = np.random.default_rng(3)
+    t = ExitTable((4, 8, 12), 16, rng.random((50, 3)), rng.random((50, 3)), rng.random(50),
+                  rng.random((50, 3)) < 0.4)
+    path = str(tmp_path / "table.npz")
+    t.save(path)
+    u = ExitTable.load(path)
+    assert u.cands == t.cands and u.n_layers == t.n_layers
+    for name in ("conf", "ent", "trace", "correct"):
+        assert np.array_equal(getattr(u, name), getattr(t, name)), name
+    assert u.correct.dtype == bool and np.array_equal(u.agreement(), t.agreement())
