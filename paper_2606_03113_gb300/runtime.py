@@ -110,7 +110,13 @@ class Engine:
         cand_arr = (C.c_int32 * max(1, len(cand)))(*cand)
         qp = None
         if qnet_params is not None:
-            self._qp = np.ascontiguousarray(qnet_params, dtype=np.float32)
+            arr = np.ascontiguousarray(qnet_params, dtype=np.float32).ravel()
+            # the library copies W1[hidden][in], b1, W2[2][hidden], b2 from this pointer
+            need = qnet_hidden * (qnet_in + 3) + 2
+            if kind == S.SSD_POLICY_LEDE and arr.size != need:
+                raise ValueError(f"qnet_params holds {arr.size} floats; a network with "
+                                 f"{qnet_in} inputs and {qnet_hidden} hidden units needs {need}")
+            self._qp = arr
             qp = self._qp.ctypes.data_as(C.POINTER(C.c_float))
         p = S.ssd_policy(kind, len(cand), C.cast(cand_arr, C.POINTER(C.c_int32)), kmax, static_l,
                          static_k, qnet_in, qnet_hidden, qp, trace_T, topk, fixed_k, conf_threshold,

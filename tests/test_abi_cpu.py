@@ -111,3 +111,19 @@ def test_struct_layouts_match_the_c_compiler(tmp_path):
         assert got[(name, "sizeof")] == C.sizeof(st), name
         for field, _ in st._fields_:
             assert got[(name, field)] == getattr(st, field).offset, (name, field)
+
+
+def test_binding_checks_the_q_network_size_before_the_call():
+    """The binding refuses a parameter array whose size does not match the
+    network's shape before the library would read past it."""
+    import numpy as np
+    from paper_2606_03113_gb300.runtime import Engine
+
+    class NoCtx:  # no device context: the check must come first
+        pass
+
+    for q_in, hidden, size in ((3, 8, 8 * 6 + 2 - 1), (257, 4, 3 * 6 + 2)):
+        with pytest.raises(ValueError):
+            Engine.set_policy(NoCtx(), S.SSD_POLICY_LEDE, cand=(1, 2), kmax=4,
+                              qnet_params=np.zeros(size, np.float32), qnet_hidden=hidden,
+                              qnet_in=q_in)
