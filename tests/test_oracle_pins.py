@@ -539,8 +539,17 @@ SMALL_GQA_BF16 = ModelShape("gqa-bf16", 4, 256, 8, 2, 32, 512, 1024, 1e-5, 50000
                             sigma=0.05, late_scale=0.2)
 
 
+# query width Hq * hd (4 x 24 = 96) unlike d (80), every dimension distinct:
+# a transposed projection or a rows/cols mix-up changes every output
+ODD_F32 = ModelShape("odd-f32", 4, 80, 4, 2, 24, 56, 72, 1e-5, 10000.0, "f32", sigma=0.05,
+                     late_scale=0.3)
+ODD_BF16 = ModelShape("odd-bf16", 4, 80, 4, 2, 24, 56, 72, 1e-5, 500000.0, "bf16", sigma=0.05,
+                      late_scale=0.3)
+
+
 @pytest.mark.parametrize("shape,l_exit", [(TINY.shape, 1), (TINY.shape, 2), (TINY.shape, 4),
-                                          (SMALL_GQA_BF16, 3), (SMALL_GQA_BF16, 4)])
+                                          (SMALL_GQA_BF16, 3), (SMALL_GQA_BF16, 4),
+                                          (ODD_BF16, 4)])
 def test_numpy_restatement_of_the_tiny_forward(shape, l_exit):
     s = shape
     ids = list(synth.prompt_ids(12, s.vocab))
@@ -551,6 +560,83 @@ def test_numpy_restatement_of_the_tiny_forward(shape, l_exit):
         for i in range(len(ids)):
             z = om.logits(h[i])
             assert np.abs(z - ref[i]).max() <= 1e-9 * np.abs(ref[i]).max(), (l_exit, i)
+    finally:
+        om.close()
+
+
+# -------------------------------------- matrix products the GPU tests check with
+
+
+def _generated(s, tid, rows, cols, sig, seed=synth.SEED_WEIGHTS, start=0):
+    """Rows of a generated matrix from the seeded generator alone (synth.h),
+    in the model's storage precision, as a float64 numpy array."""
+    if s.dtype == "bf16":
+        w = synth.bf16_bits_to_f32(synth.weights_bf16_bits(seed, tid, start, rows * cols, sig))
+    else:
+        w = synth.weights_f32(seed, tid, start, rows * cols, sig)
+    return w.astype(np.float64).reshape(rows, cols)
+
+
+def _matrices(s):
+    """(selector, tensor id of layer l, rows, cols, late-scaled) of every matrix."""
+    d, qd = s.d_model, s.n_heads * s.head_dim
+    return [(oracle.T_WQKV, lambda l: synth.layer_tid(l, synth.LT_WQKV), s.qkv_rows, d, False),
+            (oracle.T_WO, lambda l: synth.layer_tid(l, synth.LT_WO), d, qd, True),
+            (oracle.T_WGU, lambda l: synth.layer_tid(l, synth.LT_WGU), 2 * s.ffn_dim, d, False),
+            (oracle.T_WDOWN, lambda l: synth.layer_tid(l, synth.LT_WDOWN), d, s.ffn_dim, True),
+            (oracle.T_LMHEAD, lambda l: synth.TID_LMHEAD, s.vocab, d, False),
+            (oracle.T_EMBED, lambda l: synth.TID_EMBED, s.vocab, d, False)]
+
+
+@pytest.mark.parametrize("shape", [ODD_F32, ODD_BF16])
+def test_orc_matvec_every_matrix_against_numpy(shape):
+    """orc_matvec picks each matrix's own row and column counts: the product
+    equals numpy's W @ x with W taken from the generator, for every matrix
+    kind, early and late (scaled) layers, on a shape whose query width
+    differs from d."""
+    s = shape
+    om = oracle.Model(s)
+    rng = np.random.default_rng(11)
+    try:
+        for which, tid, rows, cols, late in _matrices(s):
+            for l in (0, s.n_layers - 1):
+                sig = s.sigma * (s.late_scale if late and l >= s.n_layers // 2 else 1.0)
+                W = _generated(s, tid(l), rows, cols, sig)
+                x = rng.normal(size=cols)
+                y = om.matvec(which, l, x)
+                ref = W @ x
+                assert y.shape == (rows,)
+                assert np.abs(y - ref).max() <= 1e-12 * np.abs(ref).max(), (which, l)
+    finally:
+        om.close()
+
+
+@pytest.mark.parametrize("bf16", [False, True])
+def test_orc_matvec_synth_against_numpy_and_the_model(bf16):
+    """orc_matvec_synth (the checker of the full-size products) takes row
+    row0 + r of a K-column generated matrix from flat index (row0 + r) K + k:
+    a block of rows away from the start, with K odd, equals numpy's product of
+    the generator's rows; and on every matrix of a model it equals the
+    model's own product bit for bit (same values, same order)."""
+    s = ODD_BF16 if bf16 else ODD_F32
+    rng = np.random.default_rng(5)
+    seed, tid, sig, K, row0, n = 3, 77, 0.03, 203, 37, 11
+    W = _generated(s, tid, n, K, sig, seed=seed, start=row0 * K)
+    x = rng.normal(size=K)
+    y = oracle.matvec_synth(seed, tid, sig, bf16, row0, n, x)
+    assert np.abs(y - W @ x).max() <= 1e-12 * np.abs(W @ x).max()
+    # the first row alone, and a different row0, select different rows
+    y1 = oracle.matvec_synth(seed, tid, sig, bf16, row0 + 3, 1, x)
+    assert y1[0] == y[3]
+    om = oracle.Model(s)
+    try:
+        for which, tid_l, rows, cols, late in _matrices(s):
+            for l in (0, s.n_layers - 1):
+                sc = s.sigma * (s.late_scale if late and l >= s.n_layers // 2 else 1.0)
+                x = rng.normal(size=cols)
+                ym = om.matvec(which, l, x)
+                ys = oracle.matvec_synth(synth.SEED_WEIGHTS, tid_l(l), sc, bf16, 0, rows, x)
+                assert np.array_equal(ym, ys), (which, l)
     finally:
         om.close()
 
