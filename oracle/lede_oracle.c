@@ -366,29 +366,39 @@ static void block_row(orc_sess* s, int l, int pos, double* h, double* buf) {
   }
   int group = Hq / Hkv;
   double scale = 1.0 / sqrt((double)hd);
-  for (int hh = 0; hh < Hq; ++hh) {
-    int g = hh / group;
-    const double* qh = q + (int64_t)hh * hd;
-    double mx = -INFINITY;
-    for (int t = 0; t <= pos; ++t) {
-      const double* kt = kv_row(s, l, 0, g, t);
-      double dot = 0.0;
-      for (int i = 0; i < hd; ++i) dot += qh[i] * kt[i];
-      sc[t] = dot * scale;
-      if (sc[t] > mx) mx = sc[t];
+  /* heads are independent: long contexts spread them over threads, each
+   * with its own score row (the per-head arithmetic is the same either way) */
+  int par = (int64_t)Hq * (pos + 1) * hd > (1 << 20);
+#pragma omp parallel if (par)
+  {
+    double* scr = par ? (double*)malloc(sizeof(double) * (size_t)(pos + 1)) : sc;
+#pragma omp for schedule(static)
+    for (int hh = 0; hh < Hq; ++hh) {
+      if (!scr) continue; /* out of memory: the caller sees NaN outputs */
+      int g = hh / group;
+      const double* qh = q + (int64_t)hh * hd;
+      double mx = -INFINITY;
+      for (int t = 0; t <= pos; ++t) {
+        const double* kt = kv_row(s, l, 0, g, t);
+        double dot = 0.0;
+        for (int i = 0; i < hd; ++i) dot += qh[i] * kt[i];
+        scr[t] = dot * scale;
+        if (scr[t] > mx) mx = scr[t];
+      }
+      double sum = 0.0;
+      for (int t = 0; t <= pos; ++t) {
+        scr[t] = exp(scr[t] - mx);
+        sum += scr[t];
+      }
+      double* o = att + (int64_t)hh * hd;
+      for (int i = 0; i < hd; ++i) o[i] = 0.0;
+      for (int t = 0; t <= pos; ++t) {
+        const double* vt = kv_row(s, l, 1, g, t);
+        double p = scr[t] / sum;
+        for (int i = 0; i < hd; ++i) o[i] += p * vt[i];
+      }
     }
-    double sum = 0.0;
-    for (int t = 0; t <= pos; ++t) {
-      sc[t] = exp(sc[t] - mx);
-      sum += sc[t];
-    }
-    double* o = att + (int64_t)hh * hd;
-    for (int i = 0; i < hd; ++i) o[i] = 0.0;
-    for (int t = 0; t <= pos; ++t) {
-      const double* vt = kv_row(s, l, 1, g, t);
-      double p = sc[t] / sum;
-      for (int i = 0; i < hd; ++i) o[i] += p * vt[i];
-    }
+    if (par) free(scr);
   }
   matvec(&m->wo[l], 0, d, qd, att, y);
   for (int i = 0; i < d; ++i) h[i] += y[i];
