@@ -84,13 +84,20 @@ ssd_status ssd_op_layer(ssd_ctx* ctx, int32_t kernel, int32_t layer, int32_t M, 
  * that uses it until the process exits).
  * Limits: 1 <= M <= 17 and rows <= 131072 (SSD_ERR_CAPACITY beyond), cols *
  * element size a multiple of 16 (SSD_ERR_INVALID_ARG otherwise).
+ * Device-side failure: the kernel's pipeline waits are bounded; one that gives
+ * up sets an error word (SSD error bits, 16 = a wait timed out) in the static
+ * array and leaves y_dev undefined.  With err_dev (device, one int32, may be
+ * NULL) the call enqueues, after the kernel, a copy of that word into
+ * *err_dev: 0 once the stream has reached it means y_dev holds the product.
+ * The returned status covers only the host-side checks and the launch.
  * The first call on a device looks up the array's device address and sets
  * kernel attributes; make that first call before any stream capture.  Every
- * call clears the scratch's tickets on `stream` and shares the one array, so
- * calls that overlap on the GPU (other streams, other threads) race.  Enqueued
- * on `stream`; no synchronisation; allocates nothing. */
+ * call clears the scratch's tickets and error word on `stream` and shares the
+ * one array, so calls that overlap on the GPU (other streams, other threads)
+ * race.  Enqueued on `stream`; no synchronisation; allocates nothing. */
 ssd_status ssd_gemv_noalloc(const void* W, int32_t dtype, int32_t rows, int32_t cols,
-                            const float* x_dev, int32_t M, float* y_dev, void* stream);
+                            const float* x_dev, int32_t M, float* y_dev, int32_t* err_dev,
+                            void* stream);
 
 /* Test fixture: fills dst (device, n elements of dtype) with the seeded
  * synthetic weights of tensor `tid` (see synth/synth.h): element i is

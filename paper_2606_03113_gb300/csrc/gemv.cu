@@ -1007,7 +1007,7 @@ NoAllocDevice g_noalloc_dev[64];
 
 extern "C" ssd_status ssd_gemv_noalloc(const void* W, int32_t dtype, int32_t rows, int32_t cols,
                                        const float* x_dev, int32_t M, float* y_dev,
-                                       void* stream) {
+                                       int32_t* err_dev, void* stream) {
   using namespace ssd;
   if (!W || !x_dev || !y_dev || ((uintptr_t)W & 15u) || ((uintptr_t)x_dev & 15u))
     return SSD_ERR_INVALID_ARG;
@@ -1046,9 +1046,13 @@ extern "C" ssd_status ssd_gemv_noalloc(const void* W, int32_t dtype, int32_t row
   // tickets and the error word start at zero on every call
   if (cudaMemsetAsync(B.tile_counter, 0, kNoAllocCount + kNoAllocCtl, st) != cudaSuccess)
     return SSD_ERR_CUDA;
-  return launch_gemv_plain(D, B, dtype, W, rows, cols, x_dev, M, y_dev, st) == cudaSuccess
-             ? SSD_OK
-             : SSD_ERR_CUDA;
+  if (launch_gemv_plain(D, B, dtype, W, rows, cols, x_dev, M, y_dev, st) != cudaSuccess)
+    return SSD_ERR_CUDA;
+  // the error word a bounded wait sets when it gives up, for the caller to read
+  if (err_dev && cudaMemcpyAsync(err_dev, &B.ctl->err, sizeof(int32_t), cudaMemcpyDeviceToDevice,
+                                 st) != cudaSuccess)
+    return SSD_ERR_CUDA;
+  return SSD_OK;
 }
 
 namespace ssd {

@@ -534,10 +534,22 @@ __device__ void worker_units(const TArgs& a, const Blk<TP, KIND == kKHead>& k, u
         mine[(size_t)t * 128 + srow] = grp ? v[0][2 * lt + 1] : v[0][2 * lt];
         mine[(size_t)(kMaxM + t) * 128 + srow] = grp ? v[1][2 * lt + 1] : v[1][2 * lt];
       }
-      __threadfence();
       named_sync(1, kWThreads);
-      if (tid == 0) atomicAdd(&a.B.tile_counter[tile], 1u);  // result unused: a reduction
+      if (tid == 0) red_release_gpu(&a.B.tile_counter[tile], 1u);
       return;
+    }
+    // residual kernels: the rows' previous values (written by an earlier
+    // phase or kernel), loaded while the contributors are counted in
+    float hp0[LTN], hp1[LTN];
+    if constexpr (KIND == kKResid) {
+      const int r0 = trow(g, tile, srow), r1 = trow(g, tile, srow + 128);
+#pragma unroll
+      for (int lt = 0; lt < LTN; ++lt) {
+        const int t = 2 * lt + grp;
+        const float* hm = a.B.h + (size_t)(t < M ? t : 0) * a.D.d;
+        hp0[lt] = (t < M && r0 >= 0) ? __ldcg(hm + r0) : 0.f;
+        hp1[lt] = (t < M && r1 >= 0) ? __ldcg(hm + r1) : 0.f;
+      }
     }
     if (tid == 0) {
       int contrib = 0;
@@ -561,18 +573,6 @@ __device__ void worker_units(const TArgs& a, const Blk<TP, KIND == kKHead>& k, u
     // round trips rather than one per contributor and token.  Unused slots
     // read block 0's partials (valid memory) and add zero.
     constexpr int GB = LTN <= 4 ? 4 : (LTN <= 8 ? 2 : 1);
-    // residual kernels: the rows' previous values, loaded with the partials
-    float hp0[LTN], hp1[LTN];
-    if constexpr (KIND == kKResid) {
-      const int r0 = trow(g, tile, srow), r1 = trow(g, tile, srow + 128);
-#pragma unroll
-      for (int lt = 0; lt < LTN; ++lt) {
-        const int t = 2 * lt + grp;
-        const float* hm = a.B.h + (size_t)(t < M ? t : 0) * a.D.d;
-        hp0[lt] = (t < M && r0 >= 0) ? __ldcg(hm + r0) : 0.f;
-        hp1[lt] = (t < M && r1 >= 0) ? __ldcg(hm + r1) : 0.f;
-      }
-    }
     float u0[LTN], u1[LTN];
 #pragma unroll
     for (int lt = 0; lt < LTN; ++lt) {  // b0's own partial first (0 + x: exactly x)
@@ -816,12 +816,10 @@ __global__ void __launch_bounds__(kTThreads, 1)
         for (int qq = 0; qq < 4; ++qq) part_merge(p, run[((tid & 1) * 4 + qq) * kLT + (tid >> 1)]);
         sl[(size_t)blockIdx.x * kMaxM + tid] = p;
       }
-      __threadfence();
       named_sync(1, kWThreads);
-      if (tid == 0) *sflag = atomicAdd(a.B.head_counter, 1u) == (unsigned)(g.P - 1);
+      if (tid == 0) *sflag = atom_add_acq_rel_gpu(a.B.head_counter, 1u) == (unsigned)(g.P - 1);
       named_sync(1, kWThreads);
       if (*sflag) {
-        __threadfence();
         // per row: every worker thread takes blocks tid, tid + 256, ... (the
         // running and split slots loaded together), then a shuffle tree per
         // warp and a tree over the eight warps; the order does not depend on M
@@ -1010,9 +1008,8 @@ __global__ void __launch_bounds__(kCThreads, 1)
       worker_units<TP, KIND, NORM>(a, k, tmem, u_begin, n, gi, tc, ok, pos0, M);
       gi += n;
       // this block's outputs of phase p are written: arrive
-      __threadfence();
       named_sync(1, kWThreads);
-      if (tid == 0) atomicAdd(ca.bar, 1u);
+      if (tid == 0) red_release_gpu(ca.bar, 1u);
     };
     phase(std::integral_constant<int, kKResid>{}, std::false_type{}, 0);
     phase(std::integral_constant<int, kKGateUp>{}, std::true_type{}, 1);

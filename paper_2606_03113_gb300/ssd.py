@@ -116,7 +116,7 @@ SIGNATURES = {
     "ssd_read_state": (C.c_int, [_P, _P, _P, _P, _I32, _P]),
     "ssd_op_gemv": (C.c_int, [_P, _I32, _I32, _I32, _P, _P, _P]),
     "ssd_op_layer": (C.c_int, [_P, _I32, _I32, _I32, _I32, _P]),
-    "ssd_gemv_noalloc": (C.c_int, [_P, _I32, _I32, _I32, _P, _I32, _P, _P]),
+    "ssd_gemv_noalloc": (C.c_int, [_P, _I32, _I32, _I32, _P, _I32, _P, _P, _P]),
     "ssd_synth_fill": (C.c_int, [_P, _I32, _U64, _U32, _U32, C.c_double, _P]),
     "ssd_read_probe": (C.c_int, [_P, _U64, _P, _P]),
 }
@@ -280,10 +280,11 @@ def ssd_op_layer(ctx: int, kernel: int, layer: int, M: int, pos0: int, stream_pt
 
 
 def ssd_gemv_noalloc(w_ptr: int, dtype: int, rows: int, cols: int, x_ptr: int, M: int, y_ptr: int,
-                     stream_ptr: int = 0):
-    """y = W x without a context or any device allocation (see ssd_ops.h)."""
-    _check(lib().ssd_gemv_noalloc(w_ptr, dtype, rows, cols, x_ptr, M, y_ptr, stream_ptr or None),
-           "ssd_gemv_noalloc")
+                     err_ptr: int = 0, stream_ptr: int = 0):
+    """y = W x without a context or any device allocation (see ssd_ops.h);
+    err_ptr (device int32, optional) receives the kernel's error word."""
+    _check(lib().ssd_gemv_noalloc(w_ptr, dtype, rows, cols, x_ptr, M, y_ptr, err_ptr or None,
+                                  stream_ptr or None), "ssd_gemv_noalloc")
 
 
 def ssd_synth_fill(dst_ptr: int, dtype: int, n: int, seed: int, tid: int, sigma: float,

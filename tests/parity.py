@@ -167,13 +167,21 @@ def first_token_margin(om, ids) -> float:
 def generation_parity(eng, om, w, ids, kind: str, n_new: int, tol_tok: float, tol_q: float,
                       q_val_tol: float, qp=None, l=0, k=0, kmax=None, cand=None, fixed_k=0,
                       tau=0.0, temperature=0.0, seed=0, tol_draw=0.0, tol_acc=0.0,
-                      state="paper", discard=False) -> dict:
-    """Returns decision counts; asserts on every compared decision."""
+                      state="paper", discard=False, osess=None, first_margin=None) -> dict:
+    """Returns decision counts; asserts on every compared decision.  osess:
+    an oracle session already prefilled (greedy) with ids, so that a long
+    prompt is not run through the oracle twice; first_margin: the oracle's
+    top-1/top-2 margin of the token after the prompt, when already known."""
     P = oracle_policy(kind, w, qp, l, k, kmax, cand, fixed_k, tau, temperature, seed, state,
                       discard)
-    s = om.session(eng.max_seq)
-    ofirst = s.prefill(ids, temperature=temperature, seed=seed)
-    first_margin = s.prefill_margin if temperature > 0 else None
+    if osess is not None:
+        assert temperature == 0 and osess.kv_len == len(ids)
+        s, ofirst = osess, osess.x
+    else:
+        s = om.session(eng.max_seq)
+        ofirst = s.prefill(ids, temperature=temperature, seed=seed)
+    if temperature > 0:
+        first_margin = s.prefill_margin
     otoks, logs = s.generate(P, n_new)
     set_gpu_policy(eng, kind, w, qp, l, k, kmax, cand, fixed_k, tau, temperature, seed, state,
                    discard)
@@ -183,7 +191,8 @@ def generation_parity(eng, om, w, ids, kind: str, n_new: int, tol_tok: float, to
         if temperature > 0:
             assert first_margin <= tol_draw, (gfirst, ofirst, first_margin)
         else:
-            assert first_token_margin(om, ids) <= tol_tok, (gfirst, ofirst)
+            fm = first_margin if first_margin is not None else first_token_margin(om, ids)
+            assert fm <= tol_tok, (gfirst, ofirst)
         eng.resume(seq)
     compared = total = clear_rounds = 0
     q_err = 0.0

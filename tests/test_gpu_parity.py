@@ -158,9 +158,9 @@ def test_teacher_forced_logits_and_stats(name):
                 for key in ("entropy", "conf_k", "lse", "zmax"):
                     assert abs(g[key] - sr[key]) <= tol_logit * max(1.0, abs(sr[key])), key
                 assert abs(g["pmax"] - sr["pmax"]) <= tol_logit * sr["pmax"]
-                # the top-5 list, where its gaps are clear
-                gaps = np.diff(sr["top_logit"])
-                if np.all(np.abs(gaps) > tol_tok):
+                # the top-5 list where it is unambiguous: clear gaps between the
+                # six largest logits (a tie of the 5th and 6th changes the list)
+                if np.all(-np.diff(np.sort(zr)[::-1][:6]) > tol_tok):
                     assert g["top_idx"][:5] == sr["top_idx"][:5]
     print(name, "max relative logit error", worst)
 
