@@ -338,6 +338,37 @@ def kernel_roofline(eng, w, peak: float, pos0: int, iters: int = 5, graphs: bool
     return out
 
 
+def verify_rows_probe(eng, w, ids, layers, rows, iters: int = 20) -> dict:
+    """Time of a pass over layers 1..l (embedding, the layers, one exit head)
+    for M rows at the end of the prompt, for each l and M: CUDA events on the
+    engine's stream, mean of `iters` passes after one warm-up.  The difference
+    t(l, k + 1) - t(l, 1) bounds what reusing the drafts' early-layer states
+    in verification (LayerSkip's verify reuse) could save per round: the
+    layers' weights are read once for any M, so only the per-row work and the
+    KV writes of the k drafted rows in layers 1..l* would go."""
+    import torch
+    from paper_2606_03113_gb300 import ssd as S
+    out = {}
+    n0 = len(ids) - max(rows)
+    eng.set_ar()
+    eng.prefill(ids[:n0])
+    for l in layers:
+        out[l] = {}
+        for M in rows:
+            toks = ids[n0:n0 + M]
+            S.ssd_forward_exit(eng.ctx, toks, n0, l, 5, False, w.shape.vocab)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            e0.record(eng.stream)
+            for _ in range(iters):
+                S.ssd_forward_exit(eng.ctx, toks, n0, l, 5, False, w.shape.vocab)
+            e1.record(eng.stream)
+            torch.cuda.synchronize()
+            out[l][M] = e0.elapsed_time(e1) * 1e3 / iters
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -364,6 +395,9 @@ def main():
     ap.add_argument("--kernels-only", action="store_true",
                     help="prefill, then launch each hot-path kernel eagerly over all layers "
                          "(for per-kernel ncu captures) and print their timings")
+    ap.add_argument("--verify-rows", action="store_true",
+                    help="time passes over layers 1..l for 1..kmax+1 rows (the per-round saving "
+                         "bound of reusing drafted rows' early layers in verification) and exit")
     ap.add_argument("--layers", type=int, default=0,
                     help="override the layer count (small cases for ncu --set full)")
     args = ap.parse_args()
@@ -436,6 +470,14 @@ def main():
             eng.set_lede(w, qp if q is None else q, **smp)
 
     L = w.shape.n_layers
+    if args.verify_rows:
+        lays = sorted({c for c in w.candidates} | {L})
+        rows = sorted({1, 2, 4, 8, min(w.kmax + 1, 17)})
+        r = verify_rows_probe(eng, w, ids, lays, rows)
+        if rank == 0:
+            print(json.dumps(dict(verify_rows_us=r, workload=w.name, context=len(ids))), flush=True)
+        eng.close()
+        return
     if args.kernels_only:
         eng.set_ar()
         eng.prefill(ids)

@@ -19,7 +19,8 @@
 // Each (row, head, split) writes an unnormalised partial (max, sum, output);
 // the last split block to finish a (KV head, row) pair -- a ticket per pair --
 // merges its G heads' partials in split order with the log-sum-exp rule, so
-// the result does not depend on which block finishes last.
+// the result does not depend on which block finishes last.  A block that
+// finishes several rows merges them all at once (verification passes).
 #include <math.h>
 
 #include "kernels.h"
@@ -31,6 +32,8 @@ namespace {
 
 constexpr int kAK = kAttnKeys;   // keys per split (two per lane)
 constexpr int kAThreads = 256;
+constexpr int kMergeBatch = 40;  // split partials loaded per round of the merge
+constexpr int kMergeBatch4 = 8;  // ... four dimensions each, when merging many rows
 constexpr int kAWarps = kAThreads / 32;
 
 // Stages keys [k0, k1) of the split (relative to s0) into shared memory:
@@ -75,7 +78,8 @@ __device__ __forceinline__ void stage_keys(const T* kb, const T* vb, int hd, int
 }  // namespace
 
 template <typename T>
-__global__ void __launch_bounds__(kAThreads) k_attn(Dims D, Bufs B, int layer, RowSel sel) {
+// Three blocks per SM (the shared memory of a split allows three).
+__global__ void __launch_bounds__(kAThreads, 3) k_attn(Dims D, Bufs B, int layer, RowSel sel) {
   extern __shared__ float sm[];
   const int split = blockIdx.x, g = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -84,10 +88,7 @@ __global__ void __launch_bounds__(kAThreads) k_attn(Dims D, Bufs B, int layer, R
   float* Ks = sm;                           // [kAK][hd + 1] (padded: lane-per-key reads)
   float* Vs = Ks + kAK * (hd + 1);          // [kAK][hd]
   float* Ps = Vs + kAK * hd;                // [warps][kAK] probabilities
-  float* Cw = Ps + kAWarps * kAK;           // merge: [G][nsplit] sums, then weights
-  float* Cm = Cw + (size_t)G * D.nsplit;    // merge: [G][nsplit] maxima
-  float* CL = Cm + (size_t)G * D.nsplit;    // merge: [G] denominators
-  int* last_rows = reinterpret_cast<int*>(CL + G);  // [kMaxM] rows this block merges
+  int* last_rows = reinterpret_cast<int*>(Ps + kAWarps * kAK);  // [kMaxM] rows this block merges
   __shared__ int s_nlast;
 
   const T* kv = static_cast<const T*>(B.kv) + (size_t)layer * 2 * D.Hkv * D.max_seq * hd;
@@ -164,16 +165,17 @@ __global__ void __launch_bounds__(kAThreads) k_attn(Dims D, Bufs B, int layer, R
     __syncwarp();
   }
 
-  // tickets: the last split of (g, m) merges the group's heads for row m
-  __threadfence();
-  __syncthreads();
+  // tickets: the last split of (g, m) merges the group's heads for row m.
+  // One thread per row takes the ticket with an acquire-release add after
+  // the block barrier, which publishes the block's partials and, for the
+  // last split, makes every other split's visible to the whole block.
   if (threadIdx.x == 0) s_nlast = 0;
   __syncthreads();
   if (threadIdx.x < M && threadIdx.x >= m_first) {
     const int m = threadIdx.x;
     const int nsp = (pos0 + m) / kAK + 1;
     uint32_t* cnt = B.attn_counter + (size_t)g * kMaxM + m;
-    if (atomicAdd(cnt, 1u) == (uint32_t)(nsp - 1)) {
+    if (atom_add_acq_rel_gpu(cnt, 1u) == (uint32_t)(nsp - 1)) {
       *cnt = 0u;
       last_rows[atomicAdd(&s_nlast, 1)] = m;
     }
@@ -181,60 +183,107 @@ __global__ void __launch_bounds__(kAThreads) k_attn(Dims D, Bufs B, int layer, R
   __syncthreads();
   const int nlast = s_nlast;
   if (nlast == 0) return;
-  __threadfence();
-  for (int li = 0; li < nlast; ++li) {
-    const int m = last_rows[li];
+  // merge of every row this block finishes, all rows at once (the key and
+  // value buffers are free now): (max, sum) of every (row, head, split) in
+  // one round of loads, then the weights e^{m_s - max} and denominators (a
+  // warp per (row, head), fixed lane order), then the outputs, each the
+  // splits' partials added in split order)
+  const int NS = D.nsplit;
+  float* Cm = Ks;                                  // [nlast][G][NS] maxima
+  float* Cw = Cm + (size_t)nlast * G * NS;         // [nlast][G][NS] sums, then weights
+  float* CL = Cw + (size_t)nlast * G * NS;         // [nlast][G] denominators
+  const int npr = nlast * G;
+  for (int i = threadIdx.x; i < npr * NS; i += kAThreads) {
+    const int pr = i / NS, sp = i - pr * NS;
+    const int m = last_rows[pr / G], h = pr - (pr / G) * G;
+    if (sp > (pos0 + m) / kAK) continue;
+    const size_t pidx = ((size_t)m * D.Hq + (size_t)g * G + h) * NS + sp;
+    Cm[i] = __ldcg(&B.attn_ml[2 * pidx]);
+    Cw[i] = __ldcg(&B.attn_ml[2 * pidx + 1]);
+  }
+  __syncthreads();
+  for (int pr = warp; pr < npr; pr += kAWarps) {
+    const int m = last_rows[pr / G];
     const int nsp = (pos0 + m) / kAK + 1;
-    const size_t hbase = ((size_t)m * D.Hq + (size_t)g * G) * D.nsplit;
-    // (max, sum) of every head and split: one round of loads into shared memory
-    for (int i = threadIdx.x; i < G * nsp; i += kAThreads) {
-      const int h = i / nsp, s = i - h * nsp;
-      const size_t pidx = hbase + (size_t)h * D.nsplit + s;
-      Cm[h * D.nsplit + s] = __ldcg(&B.attn_ml[2 * pidx]);
-      Cw[h * D.nsplit + s] = __ldcg(&B.attn_ml[2 * pidx + 1]);
+    const float* cm = Cm + (size_t)pr * NS;
+    float* cw = Cw + (size_t)pr * NS;
+    float gmax = -INFINITY;
+    for (int sp = lane; sp < nsp; sp += 32) gmax = fmaxf(gmax, cm[sp]);
+    gmax = warp_max(gmax);
+    float L = 0.f;
+    for (int sp = lane; sp < nsp; sp += 32) {
+      const float l = cw[sp];
+      const float w = l > 0.f ? expf(cm[sp] - gmax) : 0.f;
+      cw[sp] = w;
+      L = fmaf(w, l, L);
     }
-    __syncthreads();
-    // weights e^{m_s - max} and denominators (one warp per head, fixed lane order)
-    for (int h = warp; h < G; h += kAWarps) {
-      float gmax = -INFINITY;
-      for (int s = lane; s < nsp; s += 32) gmax = fmaxf(gmax, Cm[h * D.nsplit + s]);
-      gmax = warp_max(gmax);
-      float L = 0.f;
-      for (int s = lane; s < nsp; s += 32) {
-        const float l = Cw[h * D.nsplit + s];
-        const float w = l > 0.f ? expf(Cm[h * D.nsplit + s] - gmax) : 0.f;
-        Cw[h * D.nsplit + s] = w;
-        L = fmaf(w, l, L);
-      }
-      L = warp_sum(L);
-      if (lane == 0) CL[h] = L;
-    }
-    __syncthreads();
-    // outputs: partials of eight splits loaded per round, added in split order
-    for (int o = threadIdx.x; o < G * hd; o += kAThreads) {
-      const int h = o / hd, dd = o - h * hd;
-      const float* part = B.attn_part + (hbase + (size_t)h * D.nsplit) * hd + dd;
-      const float* w = Cw + h * D.nsplit;
+    L = warp_sum(L);
+    if (lane == 0) CL[pr] = L;
+  }
+  __syncthreads();
+  if (npr * hd <= kAThreads) {
+    // few rows: a thread per output, all splits in one round
+    for (int o = threadIdx.x; o < npr * hd; o += kAThreads) {
+      const int pr = o / hd, dd = o - pr * hd;
+      const int m = last_rows[pr / G], h = pr - (pr / G) * G;
+      const int nsp = (pos0 + m) / kAK + 1;
+      const float* w = Cw + (size_t)pr * NS;
+      const float* part = B.attn_part + (((size_t)m * D.Hq + (size_t)g * G + h) * NS) * hd + dd;
       float O = 0.f;
-      for (int sc = 0; sc < nsp; sc += 8) {
-        float pv[8];
+      for (int sc = 0; sc < nsp; sc += kMergeBatch) {
+        float pv[kMergeBatch];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) pv[j] = sc + j < nsp ? __ldcg(part + (size_t)(sc + j) * hd) : 0.f;
+        for (int j = 0; j < kMergeBatch; ++j)
+          pv[j] = sc + j < nsp ? __ldcg(part + (size_t)(sc + j) * hd) : 0.f;
 #pragma unroll
-        for (int j = 0; j < 8; ++j)
+        for (int j = 0; j < kMergeBatch; ++j)
           if (sc + j < nsp) O = fmaf(w[sc + j], pv[j], O);
       }
-      B.attn_out[(size_t)m * D.qd + (size_t)(g * G + h) * hd + dd] = O / CL[h];
+      B.attn_out[(size_t)m * D.qd + (size_t)(g * G + h) * hd + dd] = O / CL[pr];
     }
-    __syncthreads();
+  } else {
+    // many rows (verification): a warp per (row, head), four dimensions per
+    // lane; the same sum per output, fewer rounds of loads
+    for (int pr = warp; pr < npr; pr += kAWarps) {
+      const int m = last_rows[pr / G], h = pr - (pr / G) * G;
+      const int nsp = (pos0 + m) / kAK + 1;
+      const float* w = Cw + (size_t)pr * NS;
+      const float* part = B.attn_part + (((size_t)m * D.Hq + (size_t)g * G + h) * NS) * hd;
+      float* out = B.attn_out + (size_t)m * D.qd + (size_t)(g * G + h) * hd;
+      for (int d0 = 4 * lane; d0 < hd; d0 += 128) {
+        float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int sc = 0; sc < nsp; sc += kMergeBatch4) {
+          float4 pv[kMergeBatch4];
+#pragma unroll
+          for (int j = 0; j < kMergeBatch4; ++j)
+            pv[j] = sc + j < nsp
+                        ? __ldcg(reinterpret_cast<const float4*>(part + (size_t)(sc + j) * hd + d0))
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+          for (int j = 0; j < kMergeBatch4; ++j)
+            if (sc + j < nsp) {
+              const float wj = w[sc + j];
+              O.x = fmaf(wj, pv[j].x, O.x);
+              O.y = fmaf(wj, pv[j].y, O.y);
+              O.z = fmaf(wj, pv[j].z, O.z);
+              O.w = fmaf(wj, pv[j].w, O.w);
+            }
+        }
+        const float L = CL[pr];
+        *reinterpret_cast<float4*>(out + d0) = make_float4(O.x / L, O.y / L, O.z / L, O.w / L);
+      }
+    }
   }
 }
 
 size_t attn_smem(const Dims& D) {
+  // keys and values of one split (reused by the merge: maxima, weights and
+  // denominators of up to kMaxM rows x G heads x nsplit splits), the warps'
+  // probabilities, the rows this block merges
   const int G = D.Hq / D.Hkv;
-  return sizeof(float) * ((size_t)kAK * (D.hd + 1) + (size_t)kAK * D.hd + (size_t)kAWarps * kAK +
-                          2 * (size_t)G * D.nsplit + G) +
-         sizeof(int) * kMaxM;
+  const size_t kv = (size_t)kAK * (D.hd + 1) + (size_t)kAK * D.hd;
+  const size_t merge = (2 * (size_t)D.nsplit + 1) * kMaxM * G;
+  return sizeof(float) * ((kv > merge ? kv : merge) + (size_t)kAWarps * kAK) + sizeof(int) * kMaxM;
 }
 
 template <typename T>
