@@ -52,8 +52,7 @@ def measured_peaks() -> dict:
 
 # DRAM traffic of the dominant kernel from the committed ncu summaries: valid
 # only while the kernel's sources are the ones that were captured.
-TRAFFIC_PROFILES = {"k_gate_up": "k_tile_gate_up_llama2-7b.md",
-                    "k_chain(o+gate_up+down+next_qkv)": "k_chain_llama2-7b.md"}
+TRAFFIC_PROFILES = {"k_chain(o+gate_up+down+next_qkv)": "k_chain_llama2-7b.md"}
 TRAFFIC_SOURCES = ("tile.cu", "tc.cuh", "pipe.cuh", "headpart.cuh")
 
 

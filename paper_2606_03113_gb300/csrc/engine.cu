@@ -469,7 +469,17 @@ ssd_status ssd_init_model(const ssd_model_cfg* cfg, const ssd_weights* w, void* 
   ssd_ctx* x = new ssd_ctx();
   x->cfg = *cfg;
   layout(*cfg, static_cast<char*>(workspace), &x->D, &x->B);
-  x->D.num_sms = std::min(sms, kMaxBlocks);
+  // persistent grids: one block per SM of this context, all resident at once
+  // (their phase barriers and split-tile fix-ups wait on other blocks)
+  int per_sm = 1;
+  if (cfg->dtype == SSD_DTYPE_BF16) {
+    per_sm = tile_blocks_per_sm();
+    if (per_sm < 1) {
+      delete x;
+      return fail(nullptr, SSD_ERR_UNSUPPORTED, "tensor-core kernels cannot be resident on an SM");
+    }
+  }
+  x->D.num_sms = std::min(sms * std::min(per_sm, 1), kMaxBlocks);
   x->embed = w->embed;
   x->lm_head = w->lm_head;
   x->final_norm = w->final_norm;

@@ -31,6 +31,8 @@ bool encode_weight_map(CUtensorMap* m, const void* W, int rows, int cols);
 bool encode_input_map(CUtensorMap* m, const float* x, int cols, int rows, int box_rows);
 bool encode_input_maps(CUtensorMap (&m)[3], const float* x, int cols);
 cudaError_t prepare_tile_kernels();
+// Resident blocks per SM of the tensor-core kernels (0: cannot be resident).
+int tile_blocks_per_sm();
 // Floats of the tensor-core kernels' split-tile partials for `num_sms` blocks.
 size_t tile_part_floats(int num_sms);
 cudaError_t launch_tile_part(const Dims& D, const Bufs& B, const TileMaps& tm, const LayerW& w,

@@ -1154,6 +1154,25 @@ cudaError_t prepare_tile_kernels() {
   return prep_kind<kKHead, true>();
 }
 
+// Blocks of the tensor-core kernels that can be resident on one SM at once
+// (the smallest over the instances; 1 with their 200+ KB of shared memory),
+// or 0 when one cannot be: the persistent grids wait on each other's blocks
+// (phase barriers, split-tile fix-ups), so every block must be resident.
+int tile_blocks_per_sm() {
+  int lo = 1 << 30;
+  auto occ = [&](const void* fn, int threads, size_t smem) {
+    int nb = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, fn, threads, smem) != cudaSuccess) nb = 0;
+    lo = nb < lo ? nb : lo;
+  };
+  occ((const void*)k_chain<8, true>, kCThreads, TL<8, false>::total);
+  occ((const void*)k_chain<16, true>, kCThreads, TL<16, false>::total);
+  occ((const void*)k_chain<24, true>, kCThreads, TL<24, false>::total);
+  occ((const void*)k_tile<8, kKHead, true>, kTThreads, TL<8, true>::total);
+  occ((const void*)k_tile<24, kKQKV, true>, kTThreads, TL<24, false>::total);
+  return lo;
+}
+
 size_t tile_part_floats(int num_sms) { return (size_t)num_sms * 2 * 2 * kMaxM * 128; }
 
 bool encode_input_maps(CUtensorMap (&m)[3], const float* x, int cols) {
