@@ -77,6 +77,33 @@ class ExitTable:
         per candidate layer."""
         return self.correct.mean(axis=0)
 
+    def separation(self) -> dict:
+        """How well each state feature separates correct from incorrect exits
+        at each candidate: the area under the ROC curve of -C_5 and of -H
+        (a lower value meaning a more confident exit) for the event "the exit
+        token equals the full-model token" (ties count one half); 0.5 is no
+        information, 1.0 a perfect split."""
+        def auc(score, y):
+            order = np.argsort(score, kind="stable")
+            s = score[order]
+            ranks = np.empty(len(s))
+            i = 0
+            while i < len(s):  # average ranks over ties
+                j = i
+                while j + 1 < len(s) and s[j + 1] == s[i]:
+                    j += 1
+                ranks[i:j + 1] = (i + j) / 2.0 + 1.0
+                i = j + 1
+            r = np.empty(len(s))
+            r[order] = ranks
+            npos, nneg = int(y.sum()), int(len(y) - y.sum())
+            if npos == 0 or nneg == 0:
+                return float("nan")
+            return float((r[y].sum() - npos * (npos + 1) / 2.0) / (npos * nneg))
+        return {int(c): dict(conf=auc(-self.conf[:, j], self.correct[:, j]),
+                             ent=auc(-self.ent[:, j], self.correct[:, j]))
+                for j, c in enumerate(self.cands)}
+
     def save(self, path: str):
         """Writes the table (not the token sequences) as a .npz file."""
         np.savez(path, cands=np.asarray(self.cands), n_layers=self.n_layers, conf=self.conf,

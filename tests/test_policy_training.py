@@ -76,3 +76,22 @@ def test_exit_table_save_and_load_round_trip(tmp_path):
     for name in ("conf", "ent", "trace", "correct"):
         assert np.array_equal(getattr(u, name), getattr(t, name)), name
     assert u.correct.dtype == bool and np.array_equal(u.agreement(), t.agreement())
+
+
+def test_feature_separation_auc():
+    """ExitTable.separation: a feature that orders every correct exit before
+    every incorrect one scores 1, its reverse 0, a constant 0.5 (ties count
+    one half), and an unrelated feature about 0.5."""
+    rng = np.random.default_rng(3)
+    n = 400
+    correct = rng.random((n, 3)) < 0.5
+    conf = np.where(correct, 1.0, 2.0)           # column 0: lower C_5 exactly when correct
+    conf[:, 1] = np.where(correct[:, 1], 2.0, 1.0)  # column 1: the reverse
+    conf[:, 2] = rng.random(n)                    # column 2: unrelated
+    ent = np.full((n, 3), 0.7)                    # constant
+    t = P.ExitTable((4, 8, 12), 16, conf, ent, np.zeros(n), correct)
+    sep = t.separation()
+    assert sep[4]["conf"] == pytest.approx(1.0)
+    assert sep[8]["conf"] == pytest.approx(0.0)
+    assert abs(sep[12]["conf"] - 0.5) < 0.08
+    assert all(v["ent"] == pytest.approx(0.5) for v in sep.values())
