@@ -456,7 +456,8 @@ def main():
                          walk_return=round(walk["mean_return"], 4),
                          walk_exit_layer=round(walk["exit_layer"], 2),
                          hindsight_return=round(PL.oracle_walk_return(table), 4),
-                         separation_auc_conf={int(c): round(v["conf"], 3)
+                         separation_auc_conf={int(c): (round(v["conf"], 3)
+                                                       if np.isfinite(v["conf"]) else None)
                                               for c, v in table.separation().items()},
                          updates=tlog.updates, collect_s=round(t1 - t0, 1),
                          train_s=round(t2 - t1, 1))
