@@ -512,6 +512,7 @@ def main():
                         d=acc_k / max(1, sum(1 for t in traces if t["kcap"] > 0)),
                         acc_rate=sum(t["a"] for t in traces) / max(1, acc_k),
                         tokens_per_round=n_new / max(1, len(traces)),
+                        rounds_multi_draft=sum(1 for t in traces if t["k"] > 1),
                         gb_per_token=bytes_step / n_new / 1e9)
 
     # e2e through the public API with host buffers: prompt in, tokens out
